@@ -1,0 +1,480 @@
+"""Benchmark: causal attention fwd+bwd on GB300 through the C ABI (libddattn.so).
+
+Headline workload: the 1B-model bucket sweep -- H=16, d=128, 65536 tokens per
+call, L in {256, ..., 8192} with B = 65536 / L. One step = forward + backward
+of one 65536-token batch of every bucket (6 calls of each). `value` is the
+algorithmic TFLOP/s over the step (14 d H sum_seq L(L+1)/2 flops per call).
+Also reported: per-bucket ms and TFLOP/s, the document-masked 8x8192
+concat-and-chunk step (16 seeds), the 200-step curriculum stream, the
+long-context bucket (B=4, L=16384, H=32), the roofline of the dominant kernel,
+an end-to-end number through host buffers, and the fp64 oracle's throughput on
+this host's cores.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+Multi-GPU: one process per GPU under torchrun; each rank runs its own
+replica of the workload (attention has no exchange step), scaling "weak".
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2405_13226_gb300 import workloads as wl  # noqa: E402
+
+H, D = 16, 128
+T = wl.TOKENS_PER_STEP
+PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            return json.load(f), "measured"
+    return PEAKS_FALLBACK, "fallback"
+
+
+# ------------------------------------------------------------------ dist
+def dist_setup(n_gpus):
+    import torch
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    else:
+        torch.cuda.set_device(0)
+    return rank, world, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x, world):
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# ------------------------------------------------------------------ clocks
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons during a region."""
+
+    Q = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+         "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+         "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.gpu), "--query-gpu=" + self.Q,
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *a):
+        self.lines = []
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                out, _ = self.proc.communicate(timeout=5)
+            except Exception:
+                self.proc.kill()
+                out, _ = self.proc.communicate()
+            self.lines = [l for l in out.splitlines() if l.strip()]
+
+    def summary(self):
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for l in getattr(self, "lines", []):
+            f = [x.strip() for x in l.split(",")]
+            if len(f) < 7:
+                continue
+            try:
+                sm.append(float(f[0]))
+                mx = float(f[1])
+            except ValueError:
+                continue
+            for n, v in zip(names, f[3:7]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": mx, "reasons": [], "samples": 0}
+        return {"sm_mhz": float(np.median(sm)), "sm_max_mhz": mx, "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def smi_index(local: int) -> str:
+    """nvidia-smi -i argument of this process's GPU (physical index or UUID)."""
+    vis = os.environ.get("CUDA_VISIBLE_DEVICES")
+    if vis:
+        ent = [x.strip() for x in vis.split(",") if x.strip()]
+        if local < len(ent):
+            return ent[local]
+    return str(local)
+
+
+# ------------------------------------------------------------------ CPU oracle
+def oracle_sample(max_seconds=15.0, rows_cap=None):
+    """Time the fp64 oracle on slices of the bucket sweep: head h of sequence 0
+    for every bucket, h = 0, 1, ..., until `max_seconds` of CPU work."""
+    from oracle import oracle as orc
+    orc.build()
+    qb, kb, vb, gb = wl.attn_inputs(1, max(wl.BUCKETS), 4, D, seed=0)
+    done_flops, spent, parts = 0, 0.0, []
+    for h in range(4):
+        for L in wl.BUCKETS:
+            f64 = lambda x: wl.bf16_bits_to_f32(x[0, :L, h, :]).astype(np.float64)[None]
+            q, k, v, g = f64(qb), f64(kb), f64(vb), f64(gb)
+            doc = np.zeros((1, L), np.int32)
+            t0 = time.perf_counter()
+            orc.attn_fwd(q, k, v, doc, 1 / math.sqrt(D))
+            orc.attn_bwd(q, k, v, g, doc, 1 / math.sqrt(D))
+            spent += time.perf_counter() - t0
+            done_flops += wl.attn_flops(1, L, 1, D)
+            parts.append("L=%d h=%d" % (L, h))
+            if spent >= max_seconds:
+                break
+        if spent >= max_seconds:
+            break
+    threads = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
+    return {"value": done_flops / spent / 1e12, "unit": "TFLOP/s", "cores": threads, "kind": "oracle",
+            "sample": "fp64 oracle fwd+bwd on (seq 0, head h) slices of the bucket sweep, L=256..8192, "
+                      "h=0.. until %.0f s: %d slices, %.1f s, %.3g algorithmic flops" % (
+                          max_seconds, len(parts), spent, done_flops),
+            "seconds": spent}
+
+
+# ------------------------------------------------------------------ GPU helpers
+def to_dev(bits, dev):
+    import torch
+    return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16).to(dev)
+
+
+class Bucket:
+    """Buffers of one call shape; inputs are views of shared [T, H, D] tensors."""
+
+    def __init__(self, ddattn, q, k, v, g, B, L, Hh, offsets=None, ws=None):
+        import torch
+        self.dd = ddattn
+        self.B, self.L = B, L
+        shape = (B, L, Hh, D)
+        self.q, self.k, self.v, self.g = (x.view(shape) for x in (q, k, v, g))
+        self.o = torch.empty_like(self.q)
+        self.lse = torch.empty((B, Hh, L), dtype=torch.float32, device=q.device)
+        self.dq, self.dk, self.dv = (torch.empty_like(self.q) for _ in range(3))
+        self.off = offsets
+        self.desc = ddattn.make_desc(B, L, Hh, D, None, offsets)
+        self.ws = ws if ws is not None else ddattn.new_workspace(self.desc, q.device)
+        self.flops = wl.attn_flops(B, L, Hh, D, None if offsets is None else offsets.cpu().numpy())
+        self.flops_fwd = wl.attn_flops(B, L, Hh, D, None if offsets is None else offsets.cpu().numpy(), bwd=False)
+        self.flops_bwd = self.flops - self.flops_fwd
+
+    def fwd(self, stream):
+        self.dd.fwd(self.q, self.k, self.v, None, self.off, self.o, self.lse, self.ws, stream)
+
+    def bwd(self, stream, phases=None):
+        self.dd.bwd(self.q, self.k, self.v, self.o, self.g, self.lse, None, self.off, self.dq, self.dk, self.dv,
+                    self.ws, stream, phases if phases is not None else self.dd.DD_BWD_ALL)
+
+
+def run_ours(args):
+    import torch
+    from paper_2405_13226_gb300 import ddattn
+
+    rank, world, local = dist_setup(args.gpus)
+    dev = torch.device("cuda", local if world > 1 else 0)
+    peaks, peak_src = load_peaks()
+    ddattn.lib()
+    stream = torch.cuda.current_stream()
+
+    # inputs: [T, H, D] bf16 per tensor (256 MiB each, larger than L2), seeded
+    qb, kb, vb, gb = wl.attn_inputs(1, T, H, D, seed=rank)
+    q, k, v, g = (to_dev(x, dev) for x in (qb, kb, vb, gb))
+    ws = ddattn.new_workspace(ddattn.make_desc(1, T, H, D), dev)   # same size for every bucket
+    buckets = [Bucket(ddattn, q, k, v, g, T // L, L, H, ws=ws) for L in wl.BUCKETS]
+    for bk in buckets:   # one correctness-agnostic pass so every instance is loaded
+        bk.fwd(stream); bk.bwd(stream)
+    torch.cuda.synchronize()
+
+    E = lambda: torch.cuda.Event(enable_timing=True)
+    nb = len(buckets)
+    # events: per step, per bucket: [start, after fwd, after pre, after main, after post]
+    ev = [[[E() for _ in range(5)] for _ in range(nb)] for _ in range(args.steps)]
+
+    def step(evs=None):
+        for i, bk in enumerate(buckets):
+            if evs: evs[i][0].record(stream)
+            bk.fwd(stream)
+            if evs: evs[i][1].record(stream)
+            bk.bwd(stream, ddattn.DD_BWD_PRE)
+            if evs: evs[i][2].record(stream)
+            bk.bwd(stream, ddattn.DD_BWD_MAIN)
+            if evs: evs[i][3].record(stream)
+            bk.bwd(stream, ddattn.DD_BWD_POST)
+            if evs: evs[i][4].record(stream)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    barrier(world)
+    t_start, t_end = E(), E()
+    with ClockSampler(smi_index(local)) as clk:
+        torch.cuda.synchronize()
+        t_start.record(stream)
+        for s in range(args.steps):
+            step(ev[s])
+        t_end.record(stream)
+        torch.cuda.synchronize()
+    barrier(world)
+    total_ms = max_over_ranks(t_start.elapsed_time(t_end), world)
+    st = ddattn.poll_status(ws)
+    if st != 0:
+        raise RuntimeError("device status %d (%s)" % (st, ddattn.status_string(st)))
+
+    step_flops = sum(bk.flops for bk in buckets)
+    ms_per_step = total_ms / args.steps
+    value = world * step_flops * args.steps / (total_ms * 1e-3) / 1e12
+
+    per_bucket, fwd_t, main_t, main_flops = [], 0.0, 0.0, 0
+    for i, bk in enumerate(buckets):
+        ms = [ev[s][i][0].elapsed_time(ev[s][i][4]) for s in range(args.steps)]
+        f_ms = [ev[s][i][0].elapsed_time(ev[s][i][1]) for s in range(args.steps)]
+        m_ms = [ev[s][i][2].elapsed_time(ev[s][i][3]) for s in range(args.steps)]
+        b_ms = [ev[s][i][1].elapsed_time(ev[s][i][4]) for s in range(args.steps)]
+        fwd_t += sum(f_ms); main_t += sum(m_ms); main_flops += bk.flops_bwd * args.steps
+        per_bucket.append({
+            "L": bk.L, "B": bk.B, "ms": float(np.median(ms)), "fwd_ms": float(np.median(f_ms)),
+            "bwd_ms": float(np.median(b_ms)), "bwd_main_ms": float(np.median(m_ms)),
+            "tflops": bk.flops / (np.median(ms) * 1e-3) / 1e12,
+            "fwd_tflops": bk.flops_fwd / (np.median(f_ms) * 1e-3) / 1e12,
+            "bwd_main_tflops": bk.flops_bwd / (np.median(m_ms) * 1e-3) / 1e12,
+            "frac_of_measured_sustained": bk.flops / (np.median(ms) * 1e-3) / 1e12 / peaks["bf16_tflops_sustained"],
+            "min_hbm_GBps": wl.attn_min_bytes(bk.B, bk.L, H, D) / (np.median(ms) * 1e-3) / 1e9,
+        })
+    # dominant kernel over the timed region: the backward main kernel
+    main_ach = main_flops / (main_t * 1e-3) / 1e12
+    peak = peaks["bf16_tflops_sustained"]
+    roofline = {"kernel": "attn_bwd_main_kernel<128>", "bound": "tensor", "achieved": main_ach, "peak": peak,
+                "unit": "TFLOP/s", "frac": main_ach / peak, "traffic": None,
+                "peak_kind": "bf16_tflops_sustained (%s)" % peak_src,
+                "share_of_step": main_t / total_ms,
+                "fwd_kernel_tflops": sum(bk.flops_fwd for bk in buckets) * args.steps / (fwd_t * 1e-3) / 1e12,
+                "units": "10*d*H flops per live (q,k) pair per launch (backward algorithmic count)"}
+
+    extras = {}
+    if not args.quick:
+        extras = extra_workloads(ddattn, q, k, v, g, buckets, ws, stream, peaks, dev)
+    e2e = e2e_measure(ddattn, qb, kb, vb, gb, buckets, stream, dev, args, world)
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu:
+        cpu = oracle_sample(args.cpu_seconds)
+
+    line = {
+        "metric": "causal attn fwd+bwd TFLOP/s (algorithmic, 14*d*H*sum L(L+1)/2 per call) over the bucket sweep",
+        "value": value, "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "bf16 in, fp32 accumulate", "data": "synthetic (seeded N(0,1) bf16 q,k,v,dO)",
+        "config": {"workload": "bucket sweep L=256..8192, 65536 tokens per call, H=16, d=128, causal; "
+                               "step = fwd+bwd of every bucket (6 calls)",
+                   "tokens_per_call": T, "H": H, "d": D, "buckets": list(wl.BUCKETS),
+                   "l2": "inputs larger than L2 (4 x 256 MiB bf16 tensors)", "parallelism": "replicas" if world > 1 else "1 GPU"},
+        "ms_per_64k_token_step_by_bucket": {str(p["L"]): p["ms"] for p in per_bucket},
+        "per_bucket": per_bucket,
+        "roofline": roofline,
+        "cpu_baseline": cpu,
+        "e2e": e2e,
+        "gpu_launches": args.steps * nb * 4,
+        "clocks": clk.summary(),
+    }
+    line.update(extras)
+    if rank == 0:
+        print(json.dumps(line))
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+def time_calls(fn, reps, warm, stream):
+    import torch
+    for _ in range(warm):
+        fn()
+    s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    s.record(stream)
+    for _ in range(reps):
+        fn()
+    e.record(stream)
+    torch.cuda.synchronize()
+    return s.elapsed_time(e) / reps
+
+
+def extra_workloads(ddattn, q, k, v, g, buckets, ws, stream, peaks, dev):
+    import torch
+    out = {}
+    # concat-and-chunk baseline with document masking, 16 seeds
+    dm = []
+    for seed in range(16):
+        off_np = wl.concat_and_chunk_offsets(seed)
+        off = torch.from_numpy(off_np).to(dev)
+        bk = Bucket(ddattn, q, k, v, g, 8, 8192, H, offsets=off, ws=ws)
+        ms = time_calls(lambda: (bk.fwd(stream), bk.bwd(stream)), 3, 1, stream)
+        frac = wl.live_pairs(8, 8192, off_np) / wl.live_pairs(8, 8192)
+        dm.append({"seed": seed, "ms": ms, "pair_fraction": frac, "tflops": bk.flops / (ms * 1e-3) / 1e12,
+                   "segments": int(len(wl.segment_lengths(8, 8192, off_np)))})
+    dm_mean = float(np.mean([x["ms"] for x in dm]))
+    out["dm_baseline"] = {"workload": "8 chunks x 8192, H=16, d=128, document-masked, seeds 0..15",
+                          "ms_per_step_mean": dm_mean, "per_seed": dm}
+    # curriculum stream: 200 steps, L drawn proportional to DD bucket token counts
+    counts = wl.dd_bucket_tokens(0)
+    stream_L = wl.curriculum_stream(0, 200, counts)
+    by_L = {bk.L: bk for bk in buckets}
+    torch.cuda.synchronize()
+    s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    s.record(stream)
+    for L in stream_L:
+        by_L[L].fwd(stream)
+        by_L[L].bwd(stream)
+    e.record(stream)
+    torch.cuda.synchronize()
+    cur_ms = s.elapsed_time(e) / len(stream_L)
+    cur_flops = sum(by_L[L].flops for L in stream_L) / len(stream_L)
+    out["curriculum"] = {"workload": "200 steps x 65536 tokens, H=16, d=128; L ~ bucket token share",
+                         "bucket_share": {str(L): c / sum(counts.values()) for L, c in counts.items()},
+                         "ms_per_step_mean": cur_ms, "tflops": cur_flops / (cur_ms * 1e-3) / 1e12}
+    out["dd_vs_dm_step_time_ratio"] = cur_ms / dm_mean
+    out["dd_vs_dm_flop_ratio"] = cur_flops / float(np.mean([
+        wl.attn_flops(8, 8192, H, D, wl.concat_and_chunk_offsets(sd)) for sd in range(16)]))
+    # long-context bucket: B=4, L=16384, H=32, q/k x3
+    qb, kb, vb, gb = wl.attn_inputs(4, 16384, 32, D, seed=0, qk_mult=3.0)
+    lq, lk, lv, lg = (to_dev(x, dev) for x in (qb, kb, vb, gb))
+    bk = Bucket(ddattn, lq, lk, lv, lg, 4, 16384, 32)
+    ms = time_calls(lambda: (bk.fwd(stream), bk.bwd(stream)), 5, 2, stream)
+    out["long_context"] = {"workload": "B=4 x L=16384, H=32, d=128, q/k x3", "ms": ms,
+                           "tflops": bk.flops / (ms * 1e-3) / 1e12,
+                           "frac_of_measured_sustained": bk.flops / (ms * 1e-3) / 1e12 / peaks["bf16_tflops_sustained"]}
+    del lq, lk, lv, lg, bk
+    torch.cuda.empty_cache()
+    return out
+
+
+def e2e_measure(ddattn, qb, kb, vb, gb, buckets, stream, dev, args, world):
+    """Same step through the public API with host buffers: pinned host q,k,v,dO
+    copied in, and o, lse, dq, dk, dv copied out, inside the timed region."""
+    import torch
+    host_in = [torch.from_numpy(np.ascontiguousarray(x).view(np.int16)).view(torch.bfloat16).pin_memory()
+               for x in (qb, kb, vb, gb)]
+    dev_in = [torch.empty(x.shape, dtype=torch.bfloat16, device=dev) for x in host_in]
+    outs = ["o", "dq", "dk", "dv"]
+    host_out = {n: torch.empty((T, H, D), dtype=torch.bfloat16).pin_memory() for n in outs}
+    host_lse = torch.empty(T * H, dtype=torch.float32).pin_memory()
+    views = []
+    for bk in buckets:
+        sh = (bk.B, bk.L, H, D)
+        b2 = Bucket(ddattn, *dev_in, bk.B, bk.L, H, ws=bk.ws)
+        views.append(b2)
+
+    def step():
+        for b2 in views:
+            for hsrc, d in zip(host_in, dev_in):
+                d.copy_(hsrc, non_blocking=True)
+            b2.fwd(stream)
+            b2.bwd(stream)
+            for n in outs:
+                host_out[n].copy_(getattr(b2, n).view(T, H, D), non_blocking=True)
+            host_lse.copy_(b2.lse.view(-1), non_blocking=True)
+
+    steps = max(2, min(args.steps, 5))
+    for _ in range(2):
+        step()
+    torch.cuda.synchronize()
+    barrier(world)
+    s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    s.record(stream)
+    for _ in range(steps):
+        step()
+    e.record(stream)
+    torch.cuda.synchronize()
+    ms = max_over_ranks(s.elapsed_time(e), world) / steps
+    flops = sum(bk.flops for bk in buckets)
+    h2d = len(buckets) * 4 * T * H * D * 2
+    d2h = len(buckets) * (4 * T * H * D * 2 + T * H * 4)
+    return {"value": world * flops / (ms * 1e-3) / 1e12, "unit": "TFLOP/s", "ms_per_step": ms,
+            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+            "how": "pinned host q,k,v,dO -> device, fwd+bwd via C ABI, o,lse,dq,dk,dv -> pinned host, per bucket"}
+
+
+# ------------------------------------------------------------------ reference arm
+def run_reference(args):
+    """The fp64 CPU oracle as the reference arm, on the same metric and workload
+    (bounded sample per step), on this host's cores."""
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    per = max(2.0, 60.0 / max(1, args.steps + args.warmup))
+    for _ in range(args.warmup):
+        oracle_sample(per)
+    vals, secs = [], 0.0
+    for _ in range(args.steps):
+        r = oracle_sample(per)
+        vals.append(r["value"])
+        secs += r["seconds"]
+    value = float(np.mean(vals))
+    cpu = dict(r)
+    cpu["value"] = value
+    line = {"impl": "reference",
+            "metric": "causal attn fwd+bwd TFLOP/s (algorithmic, 14*d*H*sum L(L+1)/2 per call) over the bucket sweep",
+            "value": value, "unit": "TFLOP/s", "n_gpus": int(os.environ.get("WORLD_SIZE", "1")),
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": secs / args.steps * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic (seeded N(0,1) bf16 q,k,v,dO)",
+            "config": {"workload": "bucket sweep L=256..8192, 65536 tokens per call, H=16, d=128, causal; "
+                                   "each step a bounded sample of (seq 0, head h) slices"},
+            "cpu_baseline": cpu,
+            "e2e": {"value": value, "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--quick", action="store_true", help="headline sweep only")
+    ap.add_argument("--no-cpu", action="store_true", help="skip the oracle CPU baseline")
+    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

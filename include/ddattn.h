@@ -1,0 +1,113 @@
+/*
+ * ddattn.h -- C ABI of libddattn.so: causal / document-masked multi-head
+ * self-attention, forward and backward, for one training step on one GPU
+ * (hand-written sm_103a kernels: TMA, tcgen05 UMMA, TMEM accumulators).
+ *
+ * The operation (Sec. 2.2 "Variable sequence length training" and Sec. 1):
+ *   a step is B sequences of one length L. Under dataset decomposition every
+ *   sequence is cut from a single document (Sec. 2.1, property (2)), so the
+ *   mask is plain causal (query i attends to keys j <= i). Under the
+ *   concat-and-chunk baseline with document masking (Sec. 1, Sec. 3.5 "DM"),
+ *   a chunk holds several documents and query i only attends to keys j <= i
+ *   of its own document; cu_doc_offsets gives the document starts.
+ *   With s_ij = scale * <q_i, k_j> over the live keys A(i):
+ *     LSE_i = ln sum_{j in A(i)} exp(s_ij),  P_ij = exp(s_ij - LSE_i),
+ *     o_i = sum_j P_ij v_j.
+ *   Backward, given dO = dLoss/do:
+ *     D_i = <dO_i, o_i>, dS_ij = P_ij (<dO_i, v_j> - D_i),
+ *     dq_i = scale sum_j dS_ij k_j, dk_j = scale sum_i dS_ij q_i,
+ *     dv_j = sum_i P_ij dO_i.
+ *
+ * Layouts (all device memory, caller-owned, never freed or kept by the library):
+ *   q, k, v, o, dO, dq, dk, dv : bf16, [B, L, H, d] contiguous (token-major).
+ *   lse                        : fp32, [B, H, L] contiguous, natural log.
+ *   cu_doc_offsets             : int32 [n_offsets], document starts over the
+ *                                flattened B*L tokens, non-decreasing, first 0,
+ *                                last B*L. Sequence boundaries b*L always cut
+ *                                documents, listed or not. NULL = plain causal.
+ *   ws                         : workspace of dd_attn_workspace_size() bytes,
+ *                                256-byte aligned. Its first 16 bytes hold the
+ *                                device status word: zero it once before first
+ *                                use (dd_attn_clear_status). fwd and bwd may
+ *                                share one workspace sized for bwd.
+ * All data pointers must be 16-byte aligned. Calls are asynchronous and
+ * ordered on `stream` (a cudaStream_t; NULL = legacy default stream).
+ *
+ * Errors: argument checks run on the host before any launch and return
+ * DD_ERR_INVALID_ARG / DD_ERR_UNSUPPORTED / DD_ERR_WORKSPACE with nothing
+ * launched. A failed launch returns DD_ERR_CUDA. Every wait inside the
+ * kernels is bounded; a wait that expires ends the kernel and records
+ * DD_ERR_DEVICE_TIMEOUT in the workspace status word (dd_attn_poll_status).
+ * Offsets that break the rules above give undefined values but no
+ * out-of-bounds access: every derived index is clamped into the sequence.
+ */
+#ifndef DDATTN_H
+#define DDATTN_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  DD_OK = 0,
+  DD_ERR_INVALID_ARG = 1,     /* null / misaligned pointer, bad sizes */
+  DD_ERR_UNSUPPORTED = 2,     /* head dim other than 64 or 128, device not sm_103 */
+  DD_ERR_WORKSPACE = 3,       /* workspace missing or smaller than required */
+  DD_ERR_CUDA = 4,            /* a CUDA runtime call or launch failed */
+  DD_ERR_DEVICE_TIMEOUT = 5   /* a bounded device-side wait expired */
+} dd_status;
+
+typedef struct {
+  int32_t B;                       /* sequences per call (>= 1) */
+  int32_t L;                       /* tokens per sequence (>= 1; multiples of 128 are the fast path) */
+  int32_t H;                       /* heads (>= 1) */
+  int32_t d;                       /* head dim: 64 or 128 */
+  float scale;                     /* softmax scale, usually 1/sqrt(d); finite */
+  const int32_t* cu_doc_offsets;   /* DEVICE pointer or NULL (plain causal) */
+  int32_t n_offsets;               /* entries of cu_doc_offsets (>= 2 when non-NULL) */
+} dd_attn_desc;
+
+/* Workspace bytes for dd_attn_fwd (for_bwd = 0) or dd_attn_bwd (for_bwd = 1):
+ * the status word, and for bwd the fp32 dQ accumulator [B, H, L128, d] plus
+ * the per-row D_i and LSE_i*log2(e) vectors [B, H, L128], L128 = L rounded up
+ * to a multiple of 128. Returns 0 for an invalid descriptor. */
+size_t dd_attn_workspace_size(const dd_attn_desc* desc, int for_bwd);
+
+/* Forward (Sec. 2.2 step; mask per cu_doc_offsets): writes o and lse. */
+dd_status dd_attn_fwd(const dd_attn_desc* desc, const void* q, const void* k, const void* v, void* o, float* lse,
+                      void* ws, size_t ws_bytes, void* stream);
+
+/* Backward: from q, k, v, the forward's o and lse, and dO, writes dq, dk, dv
+ * (bf16, overwritten, not accumulated). Recomputes P from lse. */
+dd_status dd_attn_bwd(const dd_attn_desc* desc, const void* q, const void* k, const void* v, const void* o,
+                      const void* dO, const float* lse, void* dq, void* dk, void* dv, void* ws, size_t ws_bytes,
+                      void* stream);
+
+/* The backward as its three kernels, for callers that time or schedule them
+ * separately: DD_BWD_PRE (D_i, padded LSE, zero the dQ accumulator in ws),
+ * DD_BWD_MAIN (P recompute and the five contractions; dK, dV and the fp32 dQ
+ * accumulator), DD_BWD_POST (dq = bf16(scale * accumulator)). `phases` is a
+ * bit mask; issuing the phases in this order, with the same arguments and
+ * workspace, equals one dd_attn_bwd call (dd_attn_bwd = all three). */
+enum { DD_BWD_PRE = 1, DD_BWD_MAIN = 2, DD_BWD_POST = 4, DD_BWD_ALL = 7 };
+dd_status dd_attn_bwd_phases(const dd_attn_desc* desc, const void* q, const void* k, const void* v,
+                             const void* o, const void* dO, const float* lse, void* dq, void* dk, void* dv,
+                             void* ws, size_t ws_bytes, int phases, void* stream);
+
+/* Zero the device status word at the head of `ws` (stream-ordered). */
+dd_status dd_attn_clear_status(void* ws, void* stream);
+
+/* Synchronise the device and return the device status word of `ws`
+ * (DD_OK, or the first error a kernel recorded there). */
+dd_status dd_attn_poll_status(const void* ws);
+
+/* Static description of a status code. */
+const char* dd_status_string(dd_status s);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* DDATTN_H */

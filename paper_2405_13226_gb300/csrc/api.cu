@@ -1,0 +1,217 @@
+// Host side of the C ABI declared in include/ddattn.h: argument checks,
+// TMA tensor maps, workspace layout, launches and the device status word.
+#include <cmath>
+#include <cstdint>
+#include <cstdlib>
+#include <cudaTypedefs.h>
+
+#include "../../include/ddattn.h"
+#include "common.cuh"
+
+namespace ddattn {
+namespace {
+
+constexpr size_t kStatusBytes = 256;  // status word + padding, keeps the rest 256-aligned
+
+size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+long long round128(long long L) { return (L + 127) / 128 * 128; }
+
+dd_status check_desc(const dd_attn_desc* d) {
+  if (!d) return DD_ERR_INVALID_ARG;
+  if (d->B < 1 || d->L < 1 || d->H < 1) return DD_ERR_INVALID_ARG;
+  if (d->B > 65535 || d->H > 65535) return DD_ERR_INVALID_ARG;  // grid y/z limits
+  if (d->d != 64 && d->d != 128) return DD_ERR_UNSUPPORTED;
+  if (!std::isfinite(d->scale) || !(d->scale > 0.f)) return DD_ERR_INVALID_ARG;
+  if (d->cu_doc_offsets) {
+    if (d->n_offsets < 2 || (reinterpret_cast<uintptr_t>(d->cu_doc_offsets) & 3u)) return DD_ERR_INVALID_ARG;
+    if ((long long)d->B * d->L > 2147483647LL) return DD_ERR_INVALID_ARG;  // int32 offsets
+  }
+  return DD_OK;
+}
+
+size_t bwd_vec_bytes(const dd_attn_desc* d) {
+  return align256((size_t)d->B * d->H * round128(d->L) * sizeof(float));
+}
+size_t bwd_acc_bytes(const dd_attn_desc* d) {
+  return align256((size_t)d->B * d->H * round128(d->L) * d->d * sizeof(float));
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }
+  return fn;
+}
+
+// 4-D map over a [B, L, H, d] bf16 tensor (dims innermost first: d, H, L, B),
+// box = 64 columns x 1 head x box_rows tokens x 1 sequence, 128B swizzle.
+// Rows past L read as zeros.
+bool make_map(CUtensorMap* m, const void* ptr, const dd_attn_desc* d, int box_rows) {
+  auto enc = encode_fn();
+  if (!enc) return false;
+  cuuint64_t dims[4] = {(cuuint64_t)d->d, (cuuint64_t)d->H, (cuuint64_t)d->L, (cuuint64_t)d->B};
+  cuuint64_t strides[3] = {(cuuint64_t)d->d * 2, (cuuint64_t)d->H * d->d * 2,
+                           (cuuint64_t)d->L * d->H * d->d * 2};
+  cuuint32_t box[4] = {64, 1, (cuuint32_t)box_rows, 1};
+  cuuint32_t es[4] = {1, 1, 1, 1};
+  CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(ptr), dims, strides, box, es,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+dd_status check_device() {
+  static int checked_dev = -1;
+  static dd_status verdict = DD_OK;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return DD_ERR_CUDA;
+  if (dev != checked_dev) {
+    int major = 0, minor = 0;
+    if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess)
+      return DD_ERR_CUDA;
+    verdict = (major == 10 && minor == 3) ? DD_OK : DD_ERR_UNSUPPORTED;
+    checked_dev = dev;
+  }
+  return verdict;
+}
+
+unsigned long long wait_limit_ns() {
+  static unsigned long long v = 0;
+  if (!v) {
+    const char* e = std::getenv("DDATTN_WAIT_LIMIT_MS");
+    long long ms = e ? std::atoll(e) : 1000;
+    if (ms < 1) ms = 1;
+    v = (unsigned long long)ms * 1000000ull;
+  }
+  return v;
+}
+
+}  // namespace
+}  // namespace ddattn
+
+using namespace ddattn;
+
+extern "C" {
+
+size_t dd_attn_workspace_size(const dd_attn_desc* desc, int for_bwd) {
+  if (check_desc(desc) != DD_OK) return 0;
+  if (!for_bwd) return kStatusBytes;
+  return kStatusBytes + 2 * bwd_vec_bytes(desc) + bwd_acc_bytes(desc);
+}
+
+dd_status dd_attn_fwd(const dd_attn_desc* desc, const void* q, const void* k, const void* v, void* o, float* lse,
+                      void* ws, size_t ws_bytes, void* stream) {
+  dd_status st = check_desc(desc);
+  if (st != DD_OK) return st;
+  if (!q || !k || !v || !o || !lse) return DD_ERR_INVALID_ARG;
+  if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(o) || !aligned16(lse))
+    return DD_ERR_INVALID_ARG;
+  if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u) || ws_bytes < dd_attn_workspace_size(desc, 0))
+    return DD_ERR_WORKSPACE;
+  if ((st = check_device()) != DD_OK) return st;
+  CUtensorMap tq, tk, tv;
+  if (!make_map(&tq, q, desc, 128) || !make_map(&tk, k, desc, 128) || !make_map(&tv, v, desc, 128))
+    return DD_ERR_CUDA;
+  FwdParams p;
+  p.B = desc->B;
+  p.L = desc->L;
+  p.H = desc->H;
+  p.nqt = (desc->L + 127) / 128;
+  p.scale_log2 = desc->scale * kLog2e;
+  p.offsets = desc->cu_doc_offsets;
+  p.n_offsets = desc->cu_doc_offsets ? desc->n_offsets : 0;
+  p.o = static_cast<__nv_bfloat16*>(o);
+  p.lse = lse;
+  p.status = static_cast<int*>(ws);
+  p.timeout_ns = wait_limit_ns();
+  cudaError_t e = launch_attn_fwd(desc->d, tq, tk, tv, p, static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? DD_OK : DD_ERR_CUDA;
+}
+
+dd_status dd_attn_bwd(const dd_attn_desc* desc, const void* q, const void* k, const void* v, const void* o,
+                      const void* dO, const float* lse, void* dq, void* dk, void* dv, void* ws, size_t ws_bytes,
+                      void* stream) {
+  return dd_attn_bwd_phases(desc, q, k, v, o, dO, lse, dq, dk, dv, ws, ws_bytes, DD_BWD_ALL, stream);
+}
+
+dd_status dd_attn_bwd_phases(const dd_attn_desc* desc, const void* q, const void* k, const void* v,
+                             const void* o, const void* dO, const float* lse, void* dq, void* dk, void* dv,
+                             void* ws, size_t ws_bytes, int phases, void* stream) {
+  if (phases < 1 || phases > DD_BWD_ALL) return DD_ERR_INVALID_ARG;
+  dd_status st = check_desc(desc);
+  if (st != DD_OK) return st;
+  if (!q || !k || !v || !o || !dO || !lse || !dq || !dk || !dv) return DD_ERR_INVALID_ARG;
+  if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(o) || !aligned16(dO) || !aligned16(lse) ||
+      !aligned16(dq) || !aligned16(dk) || !aligned16(dv))
+    return DD_ERR_INVALID_ARG;
+  if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u) || ws_bytes < dd_attn_workspace_size(desc, 1))
+    return DD_ERR_WORKSPACE;
+  if ((st = check_device()) != DD_OK) return st;
+  const int bq = desc->d == 128 ? 64 : 128;
+  CUtensorMap tq, tk, tv, tdo;
+  if (!make_map(&tq, q, desc, bq) || !make_map(&tk, k, desc, 128) || !make_map(&tv, v, desc, 128) ||
+      !make_map(&tdo, dO, desc, bq))
+    return DD_ERR_CUDA;
+  uint8_t* w = static_cast<uint8_t*>(ws);
+  BwdParams p;
+  p.B = desc->B;
+  p.L = desc->L;
+  p.H = desc->H;
+  p.L128 = (int)round128(desc->L);
+  p.nkt = (desc->L + 127) / 128;
+  p.scale = desc->scale;
+  p.scale_log2 = desc->scale * kLog2e;
+  p.offsets = desc->cu_doc_offsets;
+  p.n_offsets = desc->cu_doc_offsets ? desc->n_offsets : 0;
+  p.o = static_cast<const __nv_bfloat16*>(o);
+  p.dO = static_cast<const __nv_bfloat16*>(dO);
+  p.lse = lse;
+  p.lse2_pad = reinterpret_cast<float*>(w + kStatusBytes);
+  p.delta_pad = reinterpret_cast<float*>(w + kStatusBytes + bwd_vec_bytes(desc));
+  p.dq_acc = reinterpret_cast<float*>(w + kStatusBytes + 2 * bwd_vec_bytes(desc));
+  p.dq = static_cast<__nv_bfloat16*>(dq);
+  p.dk = static_cast<__nv_bfloat16*>(dk);
+  p.dv = static_cast<__nv_bfloat16*>(dv);
+  p.status = static_cast<int*>(ws);
+  p.timeout_ns = wait_limit_ns();
+  cudaError_t e = launch_attn_bwd(desc->d, tq, tk, tv, tdo, p, phases, static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? DD_OK : DD_ERR_CUDA;
+}
+
+dd_status dd_attn_clear_status(void* ws, void* stream) {
+  if (!ws) return DD_ERR_WORKSPACE;
+  return cudaMemsetAsync(ws, 0, sizeof(int), static_cast<cudaStream_t>(stream)) == cudaSuccess ? DD_OK
+                                                                                             : DD_ERR_CUDA;
+}
+
+dd_status dd_attn_poll_status(const void* ws) {
+  if (!ws) return DD_ERR_WORKSPACE;
+  if (cudaDeviceSynchronize() != cudaSuccess) return DD_ERR_CUDA;
+  int v = 0;
+  if (cudaMemcpy(&v, ws, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess) return DD_ERR_CUDA;
+  return static_cast<dd_status>(v);
+}
+
+const char* dd_status_string(dd_status s) {
+  switch (s) {
+    case DD_OK: return "ok";
+    case DD_ERR_INVALID_ARG: return "invalid argument";
+    case DD_ERR_UNSUPPORTED: return "unsupported (head dim must be 64 or 128; device must be sm_103)";
+    case DD_ERR_WORKSPACE: return "workspace missing, misaligned or too small";
+    case DD_ERR_CUDA: return "CUDA runtime error";
+    case DD_ERR_DEVICE_TIMEOUT: return "device-side wait timed out";
+  }
+  return "unknown status";
+}
+
+}  // extern "C"

@@ -1,0 +1,340 @@
+// Causal / document-masked attention forward for sm_103a.
+//
+// One CTA computes one 128-row query tile of one (sequence, head):
+//   O = softmax(scale * Q K^T + mask) V,  LSE = ln sum exp(scale * Q K^T + mask)
+// over the live key tiles only (tile skipping from the causal diagonal and
+// the first row's document start). Warp roles:
+//   warps 0-3  softmax: thread r owns query row r = TMEM lane r. Reads the
+//              S tile from TMEM, masks (diagonal / document-edge tiles only),
+//              online max/sum in the log2 domain, writes P (bf16) to a
+//              128B-swizzled smem tile, and rescales O in TMEM when the
+//              running max grows by more than 2^8 (otherwise the stale max
+//              is kept; P <= 256 stays exact enough in bf16/fp32).
+//   warp 4     TMA producer for Q (once) and K tiles (2-stage ring); TMEM alloc.
+//   warp 5     TMA producer for V tiles (2-stage ring).
+//   warp 6     one thread issues tcgen05.mma: S[j%2] = Q K_j^T (TMEM, fp32),
+//              then O += P_{j-1} V_{j-1} (TMEM, fp32), so the tensor core
+//              computes S_{j+1} while the softmax warps work on S_j.
+#include "common.cuh"
+
+namespace ddattn {
+
+template <int D>
+struct FwdCfg {
+  static constexpr int BM = 128, BN = 128;
+  static constexpr int DB = D / 64;                    // 64-column swizzle blocks per row
+  static constexpr int Q_BLK = BM * 128;               // bytes of one [128 rows][64] block
+  static constexpr int KV_BLK = BN * 128;
+  static constexpr int Q_BYTES = DB * Q_BLK;
+  static constexpr int KV_BYTES = DB * KV_BLK;
+  static constexpr int P_BLK = BM * 128;
+  static constexpr int P_BYTES = 2 * P_BLK;            // [128 q][128 kv] bf16
+  static constexpr int OFF_Q = 0;
+  static constexpr int OFF_K = OFF_Q + Q_BYTES;
+  static constexpr int OFF_V = OFF_K + 2 * KV_BYTES;
+  static constexpr int OFF_P = OFF_V + 2 * KV_BYTES;
+  static constexpr int OFF_BAR = OFF_P + 2 * P_BYTES;
+  static constexpr int SMEM_BYTES = OFF_BAR + 256 + 1024;
+  static constexpr uint32_t TMEM_S = 0;                // S buffers at columns 0 and 128
+  static constexpr uint32_t TMEM_O = 256;              // O: D columns
+  static constexpr uint32_t TMEM_COLS = 512;
+  static constexpr int THREADS = 224;
+};
+
+struct FwdBars {
+  uint64_t q_full;
+  uint64_t k_full[2], k_empty[2], v_full[2], v_empty[2];
+  uint64_t s_full[2], s_free[2], p_full[2], p_empty[2];
+  uint64_t mma_drain;
+  uint32_t tmem_base;
+  int abort_flag;
+};
+static_assert(sizeof(FwdBars) <= 256, "barrier block");
+
+template <int D>
+__global__ void __launch_bounds__(224, 1)
+    attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                    const __grid_constant__ CUtensorMap tmV, const FwdParams p) {
+  using C = FwdCfg<D>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = align1024(smem_raw);
+  FwdBars* bars = reinterpret_cast<FwdBars*>(smem + C::OFF_BAR);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  const int m = p.nqt - 1 - blockIdx.x;  // heaviest causal tiles first
+  const int h = blockIdx.y, b = blockIdx.z;
+  const long long seq0 = (long long)b * p.L;
+  const int row0 = m * C::BM;
+  // Live key tiles [n_lo, m]: keys before the first row's document start are
+  // masked for every row of the tile (documents start in order).
+  const int ds0 = (int)(doc_start(p.offsets, p.n_offsets, seq0 + row0, seq0) - seq0);
+  const int n_lo = ds0 / C::BN;
+  const int nt = m - n_lo + 1;
+  Watchdog wd{&bars->abort_flag, p.status, p.timeout_ns};
+
+  if (threadIdx.x == 0) {
+    bars->abort_flag = 0;
+    mbar_init(&bars->q_full, 1);
+    for (int i = 0; i < 2; i++) {
+      mbar_init(&bars->k_full[i], 1);
+      mbar_init(&bars->k_empty[i], 1);
+      mbar_init(&bars->v_full[i], 1);
+      mbar_init(&bars->v_empty[i], 1);
+      mbar_init(&bars->s_full[i], 1);
+      mbar_init(&bars->s_free[i], 128);
+      mbar_init(&bars->p_full[i], 128);
+      mbar_init(&bars->p_empty[i], 1);
+    }
+    mbar_init(&bars->mma_drain, 1);
+    fence_mbar_init();
+  }
+  if (warp == 4) {
+    tmem_alloc(&bars->tmem_base, C::TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = bars->tmem_base;
+  uint8_t* sQ = smem + C::OFF_Q;
+  uint8_t* sK = smem + C::OFF_K;
+  uint8_t* sV = smem + C::OFF_V;
+  uint8_t* sP = smem + C::OFF_P;
+
+  if (warp == 4) {
+    // ---------------- Q + K producer
+    if (lane == 0) {
+      prefetch_tmap(&tmQ);
+      prefetch_tmap(&tmK);
+      mbar_arrive_expect_tx(&bars->q_full, C::Q_BYTES);
+      for (int blk = 0; blk < C::DB; blk++) tma_load_4d(sQ + blk * C::Q_BLK, &tmQ, &bars->q_full, 64 * blk, h, row0, b);
+      int issued = 0;
+      for (int j = 0; j < nt; j++) {
+        const int s = j & 1;
+        if (j >= 2 && !mbar_wait(&bars->k_empty[s], ((j >> 1) - 1) & 1, wd)) break;
+        mbar_arrive_expect_tx(&bars->k_full[s], C::KV_BYTES);
+        const int kv0 = (n_lo + j) * C::BN;
+        for (int blk = 0; blk < C::DB; blk++)
+          tma_load_4d(sK + s * C::KV_BYTES + blk * C::KV_BLK, &tmK, &bars->k_full[s], 64 * blk, h, kv0, b);
+        issued = j + 1;
+      }
+      if (*wd.abort_flag) {  // let in-flight copies land before the CTA exits
+        mbar_wait_drain(&bars->q_full, 0, wd.limit_ns);
+        for (int j = issued - 2 < 0 ? 0 : issued - 2; j < issued; j++)
+          mbar_wait_drain(&bars->k_full[j & 1], (j >> 1) & 1, wd.limit_ns);
+      }
+    }
+  } else if (warp == 5) {
+    // ---------------- V producer
+    if (lane == 0) {
+      prefetch_tmap(&tmV);
+      int issued = 0;
+      for (int j = 0; j < nt; j++) {
+        const int s = j & 1;
+        if (j >= 2 && !mbar_wait(&bars->v_empty[s], ((j >> 1) - 1) & 1, wd)) break;
+        mbar_arrive_expect_tx(&bars->v_full[s], C::KV_BYTES);
+        const int kv0 = (n_lo + j) * C::BN;
+        for (int blk = 0; blk < C::DB; blk++)
+          tma_load_4d(sV + s * C::KV_BYTES + blk * C::KV_BLK, &tmV, &bars->v_full[s], 64 * blk, h, kv0, b);
+        issued = j + 1;
+      }
+      if (*wd.abort_flag)
+        for (int j = issued - 2 < 0 ? 0 : issued - 2; j < issued; j++)
+          mbar_wait_drain(&bars->v_full[j & 1], (j >> 1) & 1, wd.limit_ns);
+    }
+  } else if (warp == 6) {
+    // ---------------- MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t idesc_s = idesc_bf16(128, 128, false, false);  // Q, K both K-major
+      constexpr uint32_t idesc_o = idesc_bf16(128, D, false, true);      // P K-major, V MN-major
+      const uint32_t aQ = smem_u32(sQ), aK = smem_u32(sK), aV = smem_u32(sV), aP = smem_u32(sP);
+      if (mbar_wait(&bars->q_full, 0, wd)) {
+        for (int j = 0; j <= nt; j++) {
+          if (j < nt) {
+            const int s = j & 1;
+            if (!mbar_wait(&bars->k_full[s], (j >> 1) & 1, wd)) break;
+            if (j >= 2 && !mbar_wait(&bars->s_free[s], ((j >> 1) - 1) & 1, wd)) break;
+            tc_fence_after();
+#pragma unroll
+            for (int ks = 0; ks < D / 16; ks++) {
+              const uint64_t da = sdesc_sw128(aQ + (ks >> 2) * C::Q_BLK + (ks & 3) * 32, 16, 1024);
+              const uint64_t db = sdesc_sw128(aK + s * C::KV_BYTES + (ks >> 2) * C::KV_BLK + (ks & 3) * 32, 16, 1024);
+              umma_bf16(tmem + C::TMEM_S + s * 128, da, db, idesc_s, ks > 0 ? 1u : 0u);
+            }
+            umma_commit(&bars->s_full[s]);
+            umma_commit(&bars->k_empty[s]);
+          }
+          if (j >= 1) {
+            const int i = j - 1, s = i & 1;
+            if (!mbar_wait(&bars->v_full[s], (i >> 1) & 1, wd)) break;
+            if (!mbar_wait(&bars->p_full[s], (i >> 1) & 1, wd)) break;
+            tc_fence_after();
+#pragma unroll
+            for (int ks = 0; ks < C::BN / 16; ks++) {
+              const uint64_t da = sdesc_sw128(aP + s * C::P_BYTES + (ks >> 2) * C::P_BLK + (ks & 3) * 32, 16, 1024);
+              const uint64_t db = sdesc_sw128(aV + s * C::KV_BYTES + ks * 2048, C::KV_BLK, 1024);
+              umma_bf16(tmem + C::TMEM_O, da, db, idesc_o, (i > 0 || ks > 0) ? 1u : 0u);
+            }
+            umma_commit(&bars->p_empty[s]);
+            umma_commit(&bars->v_empty[s]);
+          }
+        }
+      }
+      umma_commit(&bars->mma_drain);
+      mbar_wait_drain(&bars->mma_drain, 0, wd.limit_ns);
+    }
+  } else {
+    // ---------------- softmax warps 0-3: thread r <-> query row r <-> TMEM lane r
+    const int r = threadIdx.x;
+    const int row = row0 + r;
+    const int rowc = row < p.L ? row : p.L - 1;
+    const int ds = (int)(doc_start(p.offsets, p.n_offsets, seq0 + rowc, seq0) - seq0);
+    const uint32_t tl = tmem + ((uint32_t)(warp * 32) << 16);
+    const float sl2 = p.scale_log2;
+    float m_run = -INFINITY, l_run = 0.f;
+    bool ok = true;
+    for (int j = 0; j < nt && ok; j++) {
+      const int s = j & 1;
+      const int kv0 = (n_lo + j) * C::BN;
+      ok = __all_sync(0xffffffffu, mbar_wait(&bars->s_full[s], (j >> 1) & 1, wd));
+      if (!ok) break;
+      tc_fence_after();
+      uint32_t v0[32], v1[32], v2[32], v3[32];
+      tmem_ld32(tl + C::TMEM_S + s * 128 + 0, v0);
+      tmem_ld32(tl + C::TMEM_S + s * 128 + 32, v1);
+      tmem_ld32(tl + C::TMEM_S + s * 128 + 64, v2);
+      tmem_ld32(tl + C::TMEM_S + s * 128 + 96, v3);
+      tmem_ld_wait(v0);
+      tmem_ld_wait(v1);
+      tmem_ld_wait(v2);
+      tmem_ld_wait(v3);
+      tc_fence_before();
+      mbar_arrive(&bars->s_free[s]);
+      float sc[128];
+#pragma unroll
+      for (int c = 0; c < 32; c++) {
+        sc[c] = __uint_as_float(v0[c]);
+        sc[32 + c] = __uint_as_float(v1[c]);
+        sc[64 + c] = __uint_as_float(v2[c]);
+        sc[96 + c] = __uint_as_float(v3[c]);
+      }
+      if (kv0 + C::BN - 1 > row || kv0 < ds) {
+#pragma unroll
+        for (int c = 0; c < 128; c++) {
+          const int kv = kv0 + c;
+          if (kv > row || kv < ds) sc[c] = -INFINITY;
+        }
+      }
+      float mx = sc[0];
+#pragma unroll
+      for (int c = 1; c < 128; c++) mx = fmaxf(mx, sc[c]);
+      const float m_tile = mx * sl2;
+      float alpha = 1.f;
+      bool rescale = false;
+      if (m_tile > m_run + 8.f) {
+        alpha = exp2_approx(m_run - m_tile);  // 0 when m_run = -inf
+        rescale = (j > 0);
+        m_run = m_tile;
+      }
+      const float m_use = (m_run == -INFINITY) ? 0.f : m_run;
+      float rs = 0.f;
+      uint32_t pk[64];
+#pragma unroll
+      for (int c = 0; c < 64; c++) {
+        const float p0 = exp2_approx(fmaf(sc[2 * c], sl2, -m_use));
+        const float p1 = exp2_approx(fmaf(sc[2 * c + 1], sl2, -m_use));
+        rs += p0 + p1;
+        pk[c] = pack_bf16x2(p0, p1);
+      }
+      l_run = l_run * alpha + rs;
+      // P_j -> smem buffer j%2 (free once PV_{j-2} completed)
+      if (j >= 2) {
+        ok = __all_sync(0xffffffffu, mbar_wait(&bars->p_empty[s], ((j >> 1) - 1) & 1, wd));
+        if (!ok) break;
+      }
+      const uint32_t pbase = smem_u32(sP) + s * C::P_BYTES;
+#pragma unroll
+      for (int c = 0; c < 16; c++) {
+        const uint32_t addr = pbase + (c >> 3) * C::P_BLK + sw128_offset(r, c & 7);
+        st_shared_v4(addr, pk[4 * c], pk[4 * c + 1], pk[4 * c + 2], pk[4 * c + 3]);
+      }
+      fence_proxy_async_smem();
+      // O *= alpha, after PV_{j-1} landed and before PV_j is issued.
+      if (__any_sync(0xffffffffu, rescale)) {
+        ok = __all_sync(0xffffffffu, mbar_wait(&bars->p_empty[(j - 1) & 1], ((j - 1) >> 1) & 1, wd));
+        if (!ok) break;
+        tc_fence_after();
+#pragma unroll 1
+        for (int c = 0; c < D / 32; c++) {
+          uint32_t ov[32];
+          tmem_ld32(tl + C::TMEM_O + c * 32, ov);
+          tmem_ld_wait(ov);
+#pragma unroll
+          for (int e = 0; e < 32; e++) ov[e] = __float_as_uint(__uint_as_float(ov[e]) * alpha);
+          tmem_st32(tl + C::TMEM_O + c * 32, ov);
+        }
+        tmem_st_wait();
+      }
+      tc_fence_before();
+      mbar_arrive(&bars->p_full[s]);
+    }
+    // Epilogue: O / l -> bf16, LSE = (m + log2 l) * ln2.
+    if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&bars->p_empty[(nt - 1) & 1], ((nt - 1) >> 1) & 1, wd));
+    if (ok) {
+      tc_fence_after();
+      const float inv_l = l_run > 0.f ? 1.f / l_run : 0.f;
+      const float m_use = (m_run == -INFINITY) ? 0.f : m_run;
+      __nv_bfloat16* orow = p.o + (((long long)b * p.L + rowc) * p.H + h) * D;
+#pragma unroll 1
+      for (int c = 0; c < D / 32; c++) {
+        uint32_t ov[32];
+        tmem_ld32(tl + C::TMEM_O + c * 32, ov);
+        tmem_ld_wait(ov);
+        if (row < p.L) {
+          uint4* dst = reinterpret_cast<uint4*>(orow + c * 32);
+#pragma unroll
+          for (int q = 0; q < 4; q++) {
+            uint4 w;
+            w.x = pack_bf16x2(__uint_as_float(ov[8 * q + 0]) * inv_l, __uint_as_float(ov[8 * q + 1]) * inv_l);
+            w.y = pack_bf16x2(__uint_as_float(ov[8 * q + 2]) * inv_l, __uint_as_float(ov[8 * q + 3]) * inv_l);
+            w.z = pack_bf16x2(__uint_as_float(ov[8 * q + 4]) * inv_l, __uint_as_float(ov[8 * q + 5]) * inv_l);
+            w.w = pack_bf16x2(__uint_as_float(ov[8 * q + 6]) * inv_l, __uint_as_float(ov[8 * q + 7]) * inv_l);
+            dst[q] = w;
+          }
+        }
+      }
+      if (row < p.L)
+        p.lse[((long long)b * p.H + h) * p.L + row] = l_run > 0.f ? (m_use + __log2f(l_run)) * kLn2 : -INFINITY;
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 4) {
+    tc_fence_after();
+    tmem_dealloc(tmem, C::TMEM_COLS);
+  }
+}
+
+template <int D>
+static cudaError_t launch_fwd_d(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
+                                const FwdParams& p, cudaStream_t stream) {
+  using C = FwdCfg<D>;
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(attn_fwd_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_BYTES);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  dim3 grid(p.nqt, p.H, p.B);
+  attn_fwd_kernel<D><<<grid, C::THREADS, C::SMEM_BYTES, stream>>>(tq, tk, tv, p);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_attn_fwd(int d, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
+                            const FwdParams& p, cudaStream_t stream) {
+  if (d == 64) return launch_fwd_d<64>(tq, tk, tv, p, stream);
+  return launch_fwd_d<128>(tq, tk, tv, p, stream);
+}
+
+}  // namespace ddattn

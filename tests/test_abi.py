@@ -1,0 +1,78 @@
+"""The C ABI loads, exports what include/ddattn.h declares, and rejects bad
+arguments on the host before any launch (CPU only: no kernel runs here)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2405_13226_gb300 import build
+    build.build()
+    from paper_2405_13226_gb300 import ddattn
+    return ddattn
+
+
+def _declared():
+    src = open(os.path.join(ROOT, "include", "ddattn.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(dd_[a-z_]+)\s*\(", src)))
+
+
+def test_exports_every_declared_symbol(lib):
+    names = _declared()
+    assert "dd_attn_fwd" in names and "dd_attn_bwd" in names
+    L = lib.lib()
+    for n in names:
+        assert hasattr(L, n), n
+    assert set(names) == set(lib.EXPORTS)
+
+
+def test_status_strings(lib):
+    for s in range(6):
+        assert lib.status_string(s)
+    assert "timed out" in lib.status_string(lib.DD_ERR_DEVICE_TIMEOUT)
+
+
+def test_workspace_sizes(lib):
+    d = lib.make_desc(4, 256, 2, 64)
+    assert lib.workspace_size(d, for_bwd=False) == 256
+    n = lib.workspace_size(d, for_bwd=True)
+    # status + 2 padded vectors + fp32 accumulator [B, H, L128, d]
+    assert n == 256 + 2 * 4 * 2 * 256 * 4 + 4 * 2 * 256 * 64 * 4
+    ragged = lib.make_desc(3, 200, 2, 128)
+    assert lib.workspace_size(ragged, True) == 256 + 2 * 3 * 2 * 256 * 4 + 3 * 2 * 256 * 128 * 4
+    assert lib.workspace_size(lib.make_desc(1, 128, 1, 96), True) == 0       # unsupported head dim
+    assert lib.workspace_size(lib.make_desc(0, 128, 1, 64), True) == 0       # empty batch
+
+
+def _fwd(lib, desc, ptrs, ws=0x100000, ws_bytes=1 << 20):
+    q, k, v, o, lse = ptrs
+    return lib.lib().dd_attn_fwd(ctypes.byref(desc), q, k, v, o, lse, ws, ws_bytes, None)
+
+
+def test_host_validation_before_launch(lib):
+    good = [0x10000, 0x20000, 0x30000, 0x40000, 0x50000]
+    d = lib.make_desc(2, 256, 2, 128)
+    assert _fwd(lib, d, [None] + good[1:]) == lib.DD_ERR_INVALID_ARG            # null q
+    assert _fwd(lib, d, [0x10008] + good[1:]) == lib.DD_ERR_INVALID_ARG         # misaligned q
+    assert _fwd(lib, d, good, ws=None) == lib.DD_ERR_WORKSPACE                  # no workspace
+    assert _fwd(lib, d, good, ws=0x100010) == lib.DD_ERR_WORKSPACE              # workspace not 256-aligned
+    assert _fwd(lib, d, good, ws_bytes=16) == lib.DD_ERR_WORKSPACE              # workspace too small
+    assert _fwd(lib, lib.make_desc(2, 256, 2, 80), good) == lib.DD_ERR_UNSUPPORTED
+    assert _fwd(lib, lib.make_desc(2, 0, 2, 128), good) == lib.DD_ERR_INVALID_ARG
+    bad_scale = lib.make_desc(2, 256, 2, 128)
+    bad_scale.scale = float("nan")
+    assert _fwd(lib, bad_scale, good) == lib.DD_ERR_INVALID_ARG
+    bad_off = lib.make_desc(2, 256, 2, 128)
+    bad_off.cu_doc_offsets, bad_off.n_offsets = 0x60000, 1                      # fewer than 2 offsets
+    assert _fwd(lib, bad_off, good) == lib.DD_ERR_INVALID_ARG
+    L = lib.lib()
+    assert L.dd_attn_bwd(ctypes.byref(d), *good[:3], good[3], None, good[4], *good[:3], 0x100000, 1 << 30,
+                         None) == lib.DD_ERR_INVALID_ARG                         # null dO
+    assert L.dd_attn_bwd(ctypes.byref(d), *good[:3], good[3], good[3], good[4], *good[:3], 0x100000, 256,
+                         None) == lib.DD_ERR_WORKSPACE                           # bwd needs more than the status

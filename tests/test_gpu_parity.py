@@ -1,0 +1,114 @@
+"""CUDA path (through the C ABI) vs the fp64 oracle on the same seeded inputs.
+
+Tolerances (bf16 inputs, fp32 accumulation): O max|diff| <= 1e-2 and relative
+L2 <= 5e-3; dQ, dK, dV relative L2 <= 1e-2; LSE max|diff| <= 2e-3.
+Small cases compare every element; the full-size cases run the exact launch
+configuration of bench.py and compare sampled rows of selected (b, h) slices.
+"""
+import numpy as np
+import pytest
+
+from oracle import oracle as orc
+from paper_2405_13226_gb300 import workloads as wl
+
+from attn_cases import (bits_f64, check_full, check_sampled, default_scale, doc_start_rows, run_cuda, to_f64,
+                        rel_l2, TOL_GRAD_REL, TOL_O_REL)
+
+pytestmark = pytest.mark.gpu
+
+
+def _inputs(B, L, H, d, seed=0, qk_mult=1.0):
+    return wl.attn_inputs(B, L, H, d, seed=seed, qk_mult=qk_mult)
+
+
+def test_smoke_config_causal_d64():
+    """B=4, L=256, H=2, d=64, N(0,1), scale 1/sqrt(d), no document mask: every element."""
+    errs, _ = check_full(*_inputs(4, 256, 2, 64), default_scale(64))
+    print(errs)
+
+
+@pytest.mark.parametrize("B,L,H,d", [(2, 384, 2, 128), (1, 1024, 1, 128), (3, 200, 2, 128), (2, 129, 1, 64),
+                                     (1, 1, 2, 128), (1, 1, 1, 64), (2, 7, 3, 128), (1, 300, 2, 64)])
+def test_causal_ragged_and_edges(B, L, H, d):
+    errs, _ = check_full(*_inputs(B, L, H, d, seed=L), default_scale(d))
+    print(errs)
+
+
+@pytest.mark.parametrize("d", [64, 128])
+@pytest.mark.parametrize("seed", [0, 5])
+def test_document_mask_small(d, seed):
+    """Concat-and-chunk with document masking: 2 chunks x 1024 tokens."""
+    off = wl.concat_and_chunk_offsets(seed, n_chunks=2, chunk=1024)
+    errs, _ = check_full(*_inputs(2, 1024, 2, d, seed=seed), default_scale(d), off)
+    print(errs)
+
+
+def test_document_mask_ragged_offsets():
+    """Documents of 1, 2, 127, 129 ... tokens inside a ragged-length chunk."""
+    L = 700
+    off = np.array([0, 1, 3, 130, 259, 260, 600, L, L + 5, L + 200, 2 * L], dtype=np.int32)
+    errs, _ = check_full(*_inputs(2, L, 2, 128, seed=3), default_scale(128), off)
+    print(errs)
+
+
+def test_single_key_rows_bitwise():
+    """The first token of each document attends only to itself: P = 1, l = 1, so
+    o equals v bit for bit and LSE equals scale * <q_i, k_i>."""
+    off = wl.concat_and_chunk_offsets(1, n_chunks=2, chunk=1024)
+    qb, kb, vb, gb = _inputs(2, 1024, 2, 128, seed=1)
+    scale = default_scale(128)
+    o, lse, *_ = run_cuda(qb, kb, vb, gb, scale, off)
+    o_bits = o.view(__import__("torch").int16).cpu().numpy().view(np.uint16)
+    lse = lse.cpu().numpy()
+    q, k = bits_f64(qb), bits_f64(kb)
+    for (b, i) in doc_start_rows(2, 1024, off):
+        np.testing.assert_array_equal(o_bits[b, i], vb[b, i])
+        for h in range(2):
+            assert abs(lse[b, h, i] - scale * q[b, i, h] @ k[b, i, h]) < 1e-4
+
+
+def test_document_mask_equals_separate_calls():
+    """A document-masked call equals separate plain causal calls on each document."""
+    import torch
+    L = 1024
+    off = wl.concat_and_chunk_offsets(2, n_chunks=1, chunk=L)
+    qb, kb, vb, gb = _inputs(1, L, 2, 128, seed=2)
+    scale = default_scale(128)
+    full = [to_f64(t) for t in run_cuda(qb, kb, vb, gb, scale, off)]
+    for s, e in zip(off[:-1], off[1:]):
+        part = [to_f64(t) for t in run_cuda(qb[:, s:e].copy(), kb[:, s:e].copy(), vb[:, s:e].copy(),
+                                            gb[:, s:e].copy(), scale)]
+        np.testing.assert_allclose(full[0][:, s:e], part[0], atol=2e-2)
+        np.testing.assert_allclose(full[1][:, :, s:e], part[1], atol=1e-3)
+        for a, bb in zip(full[2:], part[2:]):
+            np.testing.assert_allclose(a[:, s:e], bb, atol=5e-2)
+
+
+@pytest.mark.parametrize("L", wl.BUCKETS)
+def test_bucket_sweep_full_size(L):
+    """1B-model bucket: H=16, d=128, 65536 tokens per call (B = 65536 / L)."""
+    B, H, d = wl.TOKENS_PER_STEP // L, 16, 128
+    qb, kb, vb, gb = _inputs(B, L, H, d)
+    slices = [(0, 0), (0, H - 1), (B - 1, 3), (B // 2, 9)]
+    errs = check_sampled(qb, kb, vb, gb, default_scale(d), slices, n_rand=6)
+    print(L, errs)
+
+
+@pytest.mark.parametrize("seed", [0, 7])
+def test_dm_baseline_full_size(seed):
+    """Concat-and-chunk baseline: 8 chunks x 8192, H=16, d=128, document-masked."""
+    off = wl.concat_and_chunk_offsets(seed)
+    qb, kb, vb, gb = _inputs(8, 8192, 16, 128, seed=seed)
+    gpu = run_cuda(qb, kb, vb, gb, default_scale(128), off)
+    errs = check_sampled(qb, kb, vb, gb, default_scale(128), [(0, 0), (3, 5), (7, 15)], off, n_rand=6, gpu=gpu)
+    print(errs)
+    o_bits = gpu[0].view(__import__("torch").int16).cpu().numpy().view(np.uint16)
+    for (b, i) in doc_start_rows(8, 8192, off):
+        np.testing.assert_array_equal(o_bits[b, i], vb[b, i])
+
+
+def test_long_context_full_size():
+    """B=4 x L=16384, H=32, d=128, q/k scaled x3 before bf16 rounding."""
+    qb, kb, vb, gb = _inputs(4, 16384, 32, 128, qk_mult=3.0)
+    errs = check_sampled(qb, kb, vb, gb, default_scale(128), [(0, 0), (3, 31)], n_rand=4)
+    print(errs)
