@@ -215,7 +215,8 @@ def run_ours(args):
     qb, kb, vb, gb = wl.attn_inputs(1, T, H, D, seed=rank)
     q, k, v, g = (to_dev(x, dev) for x in (qb, kb, vb, gb))
     ws = ddattn.new_workspace(ddattn.make_desc(1, T, H, D), dev)   # same size for every bucket
-    buckets = [Bucket(ddattn, q, k, v, g, T // L, L, H, ws=ws) for L in wl.BUCKETS]
+    sweep = [args.only_L] if args.only_L else list(wl.BUCKETS)
+    buckets = [Bucket(ddattn, q, k, v, g, T // L, L, H, ws=ws) for L in sweep]
     for bk in buckets:   # one correctness-agnostic pass so every instance is loaded
         bk.fwd(stream); bk.bwd(stream)
     torch.cuda.synchronize()
@@ -288,7 +289,7 @@ def run_ours(args):
     extras = {}
     if not args.quick:
         extras = extra_workloads(ddattn, q, k, v, g, buckets, ws, stream, peaks, dev)
-    e2e = e2e_measure(ddattn, qb, kb, vb, gb, buckets, stream, dev, args, world)
+    e2e = None if args.no_e2e else e2e_measure(ddattn, qb, kb, vb, gb, buckets, stream, dev, args, world)
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu:
         cpu = oracle_sample(args.cpu_seconds)
@@ -300,7 +301,7 @@ def run_ours(args):
         "dtype": "bf16 in, fp32 accumulate", "data": "synthetic (seeded N(0,1) bf16 q,k,v,dO)",
         "config": {"workload": "bucket sweep L=256..8192, 65536 tokens per call, H=16, d=128, causal; "
                                "step = fwd+bwd of every bucket (6 calls)",
-                   "tokens_per_call": T, "H": H, "d": D, "buckets": list(wl.BUCKETS),
+                   "tokens_per_call": T, "H": H, "d": D, "buckets": sweep,
                    "l2": "inputs larger than L2 (4 x 256 MiB bf16 tensors)", "parallelism": "replicas" if world > 1 else "1 GPU"},
         "ms_per_64k_token_step_by_bucket": {str(p["L"]): p["ms"] for p in per_bucket},
         "per_bucket": per_bucket,
@@ -467,6 +468,8 @@ def main():
     ap.add_argument("--quick", action="store_true", help="headline sweep only")
     ap.add_argument("--no-cpu", action="store_true", help="skip the oracle CPU baseline")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end measurement")
+    ap.add_argument("--only-L", type=int, default=0, help="run one bucket of the sweep (profiling)")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
