@@ -97,6 +97,26 @@ dd_status dd_attn_bwd_phases(const dd_attn_desc* desc, const void* q, const void
                              const void* o, const void* dO, const float* lse, void* dq, void* dk, void* dv,
                              void* ws, size_t ws_bytes, int phases, void* stream);
 
+/* Backward for callers that cannot allocate device memory: a runtime whose
+ * own allocator holds all device memory and passes this library only the
+ * tensors it owns, or a step loop under a fixed memory budget where a
+ * cudaMalloc at step time is not allowed. The paper has no counterpart; this
+ * is a library convenience. Same operation and arguments as dd_attn_bwd, but
+ * no workspace: it uses a scratch array of DD_NOALLOC_SCRATCH_BYTES that the
+ * library keeps in device global memory (every GPU that loads the library
+ * holds it until the process exits). Sizes whose bwd workspace
+ * (dd_attn_workspace_size(desc, 1)) exceeds that return DD_ERR_WORKSPACE with
+ * nothing launched. It calls no cudaMalloc / cudaFree. The first call on a
+ * device looks up the array's device address (make it before any stream
+ * capture). All calls share the array: calls whose kernels overlap on the GPU
+ * race, so order them on one stream. device_status (device memory, may be
+ * NULL) receives this call's device status word (0, or
+ * DD_ERR_DEVICE_TIMEOUT), copied on `stream` after the backward. */
+#define DD_NOALLOC_SCRATCH_BYTES ((size_t)32 << 20)
+dd_status dd_attn_bwd_noalloc(const dd_attn_desc* desc, const void* q, const void* k, const void* v,
+                              const void* o, const void* dO, const float* lse, void* dq, void* dk, void* dv,
+                              int32_t* device_status, void* stream);
+
 /* Zero the device status word at the head of `ws` (stream-ordered). */
 dd_status dd_attn_clear_status(void* ws, void* stream);
 

@@ -32,8 +32,9 @@ class Desc(ctypes.Structure):
 
 _lib = None
 
-EXPORTS = ("dd_attn_workspace_size", "dd_attn_fwd", "dd_attn_bwd", "dd_attn_bwd_phases", "dd_attn_clear_status",
-           "dd_attn_poll_status", "dd_status_string")
+EXPORTS = ("dd_attn_workspace_size", "dd_attn_fwd", "dd_attn_bwd", "dd_attn_bwd_phases", "dd_attn_bwd_noalloc",
+           "dd_attn_clear_status", "dd_attn_poll_status", "dd_status_string")
+NOALLOC_SCRATCH_BYTES = 32 << 20
 DD_BWD_PRE, DD_BWD_MAIN, DD_BWD_POST, DD_BWD_ALL = 1, 2, 4, 7
 
 
@@ -55,6 +56,8 @@ def lib() -> ctypes.CDLL:
         L.dd_attn_bwd.restype = i32
         L.dd_attn_bwd_phases.argtypes = [dp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, i32, vp]
         L.dd_attn_bwd_phases.restype = i32
+        L.dd_attn_bwd_noalloc.argtypes = [dp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp]
+        L.dd_attn_bwd_noalloc.restype = i32
         L.dd_attn_clear_status.argtypes = [vp, vp]
         L.dd_attn_clear_status.restype = i32
         L.dd_attn_poll_status.argtypes = [vp]
