@@ -157,7 +157,7 @@ dd_status dd_attn_bwd_phases(const dd_attn_desc* desc, const void* q, const void
   if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u) || ws_bytes < dd_attn_workspace_size(desc, 1))
     return DD_ERR_WORKSPACE;
   if ((st = check_device()) != DD_OK) return st;
-  const int bq = desc->d == 128 ? 64 : 128;
+  const int bq = 128;  // query rows per backward step (both head dims)
   CUtensorMap tq, tk, tv, tdo;
   if (!make_map(&tq, q, desc, bq) || !make_map(&tk, k, desc, 128) || !make_map(&tv, v, desc, 128) ||
       !make_map(&tdo, dO, desc, bq))

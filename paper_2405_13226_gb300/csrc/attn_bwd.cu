@@ -4,7 +4,8 @@
 //   attn_bwd_pre   D_i = <dO_i, o_i> and LSE_i*log2(e) into padded per-row
 //                  vectors (rows past L: D = 0, LSE = +inf so P = 0), and
 //                  zero the fp32 dQ accumulator.
-//   attn_bwd_main  one CTA per 128-key tile of one (sequence, head). It keeps
+//   attn_bwd_main  (d = 64 here; d = 128 in attn_bwd_d128.cu)
+//                  one CTA per 128-key tile of one (sequence, head). It keeps
 //                  K, V in smem and dK, dV in TMEM, and walks the live query
 //                  tiles (diagonal .. end of the last key's document):
 //                    S^T  = K Q^T            (TMEM)  -> P^T = exp2(S^T*scale*log2e - LSE*log2e)
@@ -68,17 +69,6 @@ struct BwdBars {
   int abort_flag;
 };
 static_assert(sizeof(BwdBars) <= 256, "barrier block");
-
-__device__ __forceinline__ void named_bar_sync(int id, int count) {
-  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
-}
-
-__device__ __forceinline__ void bulk_reduce_add_f32(float* gdst, const void* ssrc, uint32_t bytes) {
-  asm volatile("cp.reduce.async.bulk.global.shared::cta.bulk_group.add.f32 [%0], [%1], %2;" ::"l"(
-                   reinterpret_cast<uint64_t>(gdst)),
-               "r"(smem_u32(ssrc)), "r"(bytes)
-               : "memory");
-}
 
 // ------------------------------------------------------------------ pre
 // One group of d/8 threads per (b, i, h) row, rows in memory order.
@@ -498,7 +488,7 @@ static cudaError_t launch_bwd_d(const CUtensorMap& tq, const CUtensorMap& tk, co
                                 const CUtensorMap& tdo, const BwdParams& p, int phases, cudaStream_t stream) {
   using C = BwdCfg<D>;
   static bool attr_set = false;
-  if (!attr_set) {
+  if (!attr_set && D != 128) {
     cudaError_t e =
         cudaFuncSetAttribute(attn_bwd_main_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_BYTES);
     if (e != cudaSuccess) return e;
@@ -519,9 +509,13 @@ static cudaError_t launch_bwd_d(const CUtensorMap& tq, const CUtensorMap& tk, co
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
   if (phases & 2) {
-    dim3 grid(p.nkt, p.H, p.B);
-    attn_bwd_main_kernel<D><<<grid, C::THREADS, C::SMEM_BYTES, stream>>>(tq, tk, tv, tdo, p);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    if constexpr (D == 128) {
+      if ((e = launch_attn_bwd_main_d128(tq, tk, tv, tdo, p, stream)) != cudaSuccess) return e;
+    } else {
+      dim3 grid(p.nkt, p.H, p.B);
+      attn_bwd_main_kernel<D><<<grid, C::THREADS, C::SMEM_BYTES, stream>>>(tq, tk, tv, tdo, p);
+      if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    }
   }
   if (phases & 4) {
     attn_bwd_post_kernel<D><<<ew_blocks, 256, 0, stream>>>(p);

@@ -1,0 +1,443 @@
+// Attention backward main kernel for head dim 128 on sm_103a.
+//
+// One CTA per 128-key tile of one (sequence, head), walking the live 128-row
+// query tiles from the diagonal to the end of the tile's last document (the
+// backward counterpart of the forward's tile skipping). Per query step i:
+//   S^T  = K Q_i^T            P^T  = exp2(S^T * scale * log2e - LSE_i * log2e)  (masked)
+//   dP^T = V dO_i^T           dS^T = P^T (dP^T - D_i)
+//   dV  += P^T dO_i           dK  += dS^T Q_i           dQ_i^T = K^T dS^T
+// All five contractions are M = 128, N = 128 UMMAs issued by one thread: an
+// instruction costs about the same for any N <= 256, so 128-row query steps
+// give each instruction twice the work of 64-row steps.
+//
+// TMEM (512 columns): two 128-column regions R[0], R[1] whose roles alternate
+// every step (A = R[i % 2], B = R[(i + 1) % 2]):
+//   A: S^T (fp32) -> P^T (bf16 pairs over its first 64 columns, A operand of
+//      dV) -> dQ^T (fp32, after dV has read P^T) -> dP^T of step i + 1
+//   B: dP^T (fp32) -> S^T of step i + 1 (as soon as dP^T is in registers)
+//   dV [256,384), dK [384,512) accumulate over the steps.
+// The tensor core runs dV_i, S_{i+1}, dK_i, dQ^T_i, dP_{i+1}, dV_{i+1}, ... so
+// that P of step i + 1 is computed while dK_i, dQ^T_i and dP_{i+1} run.
+//
+// smem: K, V resident; Q, dO, LSE, D in 2 stages. After dV_i (and dP_i) have
+// read dO_i, its buffer receives dS^T_i (bf16, [128 keys][128 queries],
+// 128B-swizzled): the A operand of dK_i (K-major view) and the B operand of
+// dQ^T_i (MN-major view). Warps 4-7 drain dQ^T in four [32 queries x 128] fp32
+// quarters staged in smem, each one cp.reduce.async.bulk .add.f32 into the
+// contiguous accumulator rows (a direct red.global per element was measured
+// slower: its load/store traffic delays the P/dS warps on the same SM).
+//
+// Warp roles: 0-3 P/dS (thread r <-> key row r <-> TMEM lane r) and the dV
+// epilogue; 4-7 dQ drain and the dK epilogue; 8 TMA producer (and TMEM owner);
+// 9 issues tcgen05.mma.
+#include "common.cuh"
+
+namespace ddattn {
+
+struct Bwd128 {
+  static constexpr int D = 128, BN = 128, BQ = 128;
+  static constexpr int BLK = 128 * 128;                  // [128 rows][64] bf16, 128B swizzle
+  static constexpr int TILE = 2 * BLK;                   // [128 rows][128] bf16
+  static constexpr int OFF_K = 0;
+  static constexpr int OFF_V = OFF_K + TILE;
+  static constexpr int OFF_Q = OFF_V + TILE;             // 2 stages
+  static constexpr int OFF_DO = OFF_Q + 2 * TILE;        // 2 stages (dO, then dS^T)
+  static constexpr int OFF_STG = OFF_DO + 2 * TILE;      // dQ staging quarter
+  static constexpr int STG_BYTES = 32 * D * 4;
+  static constexpr int OFF_LSE = OFF_STG + STG_BYTES;    // [2][128] fp32
+  static constexpr int OFF_DEL = OFF_LSE + 2 * BQ * 4;   // [2][128] fp32
+  static constexpr int OFF_BAR = OFF_DEL + 2 * BQ * 4;
+  static constexpr int SMEM_BYTES = OFF_BAR + 256 + 1024;
+  static constexpr uint32_t TM_R = 0, TM_DV = 256, TM_DK = 384;  // R[k] at TM_R + 128 k
+  static constexpr int THREADS = 320;
+};
+
+struct Bwd128Bars {
+  uint64_t kv_full;
+  uint64_t q_full[2], q_empty[2];
+  uint64_t s_full, dp_full, p_full, dp_read, dss_full, dv_done, dq_full, r_free;
+  uint64_t mma_done;
+  uint32_t tmem_base;
+  int abort_flag;
+};
+static_assert(sizeof(Bwd128Bars) <= 256, "barrier block");
+
+__global__ void __launch_bounds__(320, 1)
+    attn_bwd_main_d128_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                              const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmDO,
+                              const BwdParams p) {
+  using C = Bwd128;
+  constexpr int D = C::D, BQ = C::BQ;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = align1024(smem_raw);
+  Bwd128Bars* bars = reinterpret_cast<Bwd128Bars*>(smem + C::OFF_BAR);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  const int n = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
+  const long long seq0 = (long long)b * p.L;
+  const int kv0 = n * C::BN;
+  const int kv_last = min(kv0 + C::BN - 1, p.L - 1);
+  // Live query tiles: from the diagonal to the end of the last key's document.
+  const int de_last = (int)(doc_end(p.offsets, p.n_offsets, seq0 + kv_last, seq0 + p.L) - seq0);
+  const int m_lo = kv0 / BQ;
+  const int m_hi = (de_last - 1) / BQ;
+  const int nq = m_hi - m_lo + 1;
+  Watchdog wd{&bars->abort_flag, p.status, p.timeout_ns};
+
+  if (threadIdx.x == 0) {
+    bars->abort_flag = 0;
+    mbar_init(&bars->kv_full, 1);
+    for (int i = 0; i < 2; i++) {
+      mbar_init(&bars->q_full[i], 1);
+      mbar_init(&bars->q_empty[i], 1);
+    }
+    mbar_init(&bars->s_full, 1);
+    mbar_init(&bars->dp_full, 1);
+    mbar_init(&bars->p_full, 128);
+    mbar_init(&bars->dp_read, 128);
+    mbar_init(&bars->dss_full, 128);
+    mbar_init(&bars->dv_done, 1);
+    mbar_init(&bars->dq_full, 1);
+    mbar_init(&bars->r_free, 128);
+    mbar_init(&bars->mma_done, 1);
+    fence_mbar_init();
+  }
+  if (warp == 8) {
+    tmem_alloc(&bars->tmem_base, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = bars->tmem_base;
+  uint8_t* sK = smem + C::OFF_K;
+  uint8_t* sV = smem + C::OFF_V;
+  uint8_t* sQ = smem + C::OFF_Q;
+  uint8_t* sDO = smem + C::OFF_DO;
+  float* sSTG = reinterpret_cast<float*>(smem + C::OFF_STG);
+  float* sLSE = reinterpret_cast<float*>(smem + C::OFF_LSE);
+  float* sDEL = reinterpret_cast<float*>(smem + C::OFF_DEL);
+  const long long vec0 = ((long long)b * p.H + h) * p.L128;  // row 0 of this (b, h) in the padded vectors
+
+  if (warp == 8) {
+    // ---------------- TMA producer
+    if (lane == 0) {
+      prefetch_tmap(&tmQ);
+      prefetch_tmap(&tmK);
+      prefetch_tmap(&tmV);
+      prefetch_tmap(&tmDO);
+      mbar_arrive_expect_tx(&bars->kv_full, 2 * C::TILE);
+      for (int blk = 0; blk < 2; blk++) {
+        tma_load_4d(sK + blk * C::BLK, &tmK, &bars->kv_full, 64 * blk, h, kv0, b);
+        tma_load_4d(sV + blk * C::BLK, &tmV, &bars->kv_full, 64 * blk, h, kv0, b);
+      }
+      int issued = 0;
+      for (int i = 0; i < nq; i++) {
+        const int s = i & 1;
+        const int q0 = (m_lo + i) * BQ;
+        if (i >= 2 && !mbar_wait(&bars->q_empty[s], ((i >> 1) - 1) & 1, wd)) break;
+        mbar_arrive_expect_tx(&bars->q_full[s], 2 * C::TILE + 2 * BQ * 4);
+        for (int blk = 0; blk < 2; blk++) {
+          tma_load_4d(sQ + s * C::TILE + blk * C::BLK, &tmQ, &bars->q_full[s], 64 * blk, h, q0, b);
+          tma_load_4d(sDO + s * C::TILE + blk * C::BLK, &tmDO, &bars->q_full[s], 64 * blk, h, q0, b);
+        }
+        bulk_load(sLSE + s * BQ, p.lse2_pad + vec0 + q0, BQ * 4, &bars->q_full[s]);
+        bulk_load(sDEL + s * BQ, p.delta_pad + vec0 + q0, BQ * 4, &bars->q_full[s]);
+        issued = i + 1;
+      }
+      if (*wd.abort_flag) {  // let in-flight copies land before the CTA exits
+        mbar_wait_drain(&bars->kv_full, 0, wd.limit_ns);
+        for (int i = issued - 2 < 0 ? 0 : issued - 2; i < issued; i++)
+          mbar_wait_drain(&bars->q_full[i & 1], (i >> 1) & 1, wd.limit_ns);
+      }
+    }
+  } else if (warp == 9) {
+    // ---------------- MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t id_s = idesc_bf16(128, 128, false, false);  // K / V rows x Q / dO rows (K-major)
+      constexpr uint32_t id_kv = idesc_bf16(128, 128, false, true);  // P^T (TMEM) / dS^T (smem) x dO / Q (MN-major)
+      constexpr uint32_t id_dq = idesc_bf16(128, 128, true, true);   // K^T (MN-major) x dS^T (MN-major)
+      const uint32_t aK = smem_u32(sK), aV = smem_u32(sV), aQ = smem_u32(sQ), aDO = smem_u32(sDO);
+      bool ok = mbar_wait(&bars->kv_full, 0, wd) && mbar_wait(&bars->q_full[0], 0, wd);
+      auto issue_s = [&](int j, uint32_t reg) {  // S^T_j = K Q_j^T into region `reg`
+        const uint32_t qs = aQ + (j & 1) * C::TILE;
+#pragma unroll
+        for (int ks = 0; ks < 8; ks++) {
+          const uint32_t off = (ks >> 2) * C::BLK + (ks & 3) * 32;
+          umma_bf16(tmem + reg, sdesc_sw128(aK + off, 16, 1024), sdesc_sw128(qs + off, 16, 1024), id_s,
+                    ks > 0 ? 1u : 0u);
+        }
+        umma_commit(&bars->s_full);
+      };
+      auto issue_dp = [&](int j, uint32_t reg) {  // dP^T_j = V dO_j^T into region `reg`
+        const uint32_t os = aDO + (j & 1) * C::TILE;
+#pragma unroll
+        for (int ks = 0; ks < 8; ks++) {
+          const uint32_t off = (ks >> 2) * C::BLK + (ks & 3) * 32;
+          umma_bf16(tmem + reg, sdesc_sw128(aV + off, 16, 1024), sdesc_sw128(os + off, 16, 1024), id_s,
+                    ks > 0 ? 1u : 0u);
+        }
+        umma_commit(&bars->dp_full);
+      };
+      if (ok) {
+        tc_fence_after();
+        issue_s(0, C::TM_R);
+        issue_dp(0, C::TM_R + 128);
+      }
+      for (int i = 0; ok && i < nq; i++) {
+        const int s = i & 1;
+        const uint32_t rA = C::TM_R + (uint32_t)(i & 1) * 128, rB = C::TM_R + (uint32_t)((i + 1) & 1) * 128;
+        const uint32_t qs = aQ + s * C::TILE, os = aDO + s * C::TILE;
+        // dV += P^T dO  (A: P^T in region A, 8 columns per 16 queries)
+        if (!(ok = mbar_wait(&bars->p_full, i & 1, wd))) break;
+        tc_fence_after();
+#pragma unroll
+        for (int ks = 0; ks < 8; ks++)
+          umma_bf16_ts(tmem + C::TM_DV, tmem + rA + ks * 8, sdesc_sw128(os + ks * 2048, C::BLK, 1024), id_kv,
+                       (i > 0 || ks > 0) ? 1u : 0u);
+        umma_commit(&bars->dv_done);
+        // S^T_{i+1} into region B as soon as dP^T_i has been read out of it.
+        if (i + 1 < nq) {
+          if (!(ok = mbar_wait(&bars->q_full[(i + 1) & 1], ((i + 1) >> 1) & 1, wd) &&
+                     mbar_wait(&bars->dp_read, i & 1, wd)))
+            break;
+          tc_fence_after();
+          issue_s(i + 1, rB);
+        }
+        // dK += dS^T Q  (A: dS^T in this stage's dO buffer, K-major view)
+        if (!(ok = mbar_wait(&bars->dss_full, i & 1, wd))) break;
+        tc_fence_after();
+#pragma unroll
+        for (int ks = 0; ks < 8; ks++) {
+          const uint32_t off = (ks >> 2) * C::BLK + (ks & 3) * 32;
+          umma_bf16(tmem + C::TM_DK, sdesc_sw128(os + off, 16, 1024), sdesc_sw128(qs + ks * 2048, C::BLK, 1024),
+                    id_kv, (i > 0 || ks > 0) ? 1u : 0u);
+        }
+        // dQ^T = K^T dS^T into region A (dV_i has finished reading P^T there:
+        // dss_full is only raised after dv_done).
+        tc_fence_after();
+#pragma unroll
+        for (int ks = 0; ks < 8; ks++)
+          umma_bf16(tmem + rA, sdesc_sw128(aK + ks * 2048, C::BLK, 1024), sdesc_sw128(os + ks * 2048, C::BLK, 1024),
+                    id_dq, ks > 0 ? 1u : 0u);
+        umma_commit(&bars->dq_full);
+        umma_commit(&bars->q_empty[s]);
+        // dP^T_{i+1} into region A once the drain has read dQ^T_i out of it.
+        if (i + 1 < nq) {
+          if (!(ok = mbar_wait(&bars->r_free, i & 1, wd))) break;
+          tc_fence_after();
+          issue_dp(i + 1, rA);
+        }
+      }
+      umma_commit(&bars->mma_done);
+      mbar_wait_drain(&bars->mma_done, 0, wd.limit_ns);
+    }
+  } else if (warp < 4) {
+    // ---------------- P / dS warps
+    const int r = threadIdx.x;
+    const int kv = kv0 + r;
+    const int kvc = kv < p.L ? kv : p.L - 1;
+    const int de = (int)(doc_end(p.offsets, p.n_offsets, seq0 + kvc, seq0 + p.L) - seq0);
+    const uint32_t tl = tmem + ((uint32_t)(warp * 32) << 16);
+    const float sl2 = p.scale_log2;
+    bool ok = true;
+    for (int i = 0; i < nq && ok; i++) {
+      const int s = i & 1;
+      const int q0 = (m_lo + i) * BQ;
+      const uint32_t rA = C::TM_R + (uint32_t)(i & 1) * 128, rB = C::TM_R + (uint32_t)((i + 1) & 1) * 128;
+      ok = __all_sync(0xffffffffu,
+                      mbar_wait(&bars->s_full, i & 1, wd) && mbar_wait(&bars->q_full[s], (i >> 1) & 1, wd));
+      if (!ok) break;
+      tc_fence_after();
+      const float4* lse4 = reinterpret_cast<const float4*>(sLSE + s * BQ);
+      const float4* del4 = reinterpret_cast<const float4*>(sDEL + s * BQ);
+      const bool need_mask = (q0 < kv) || (q0 + BQ > de);
+      // P^T packed as bf16 pairs: pa = queries 0..63, pb = queries 64..127.
+      uint32_t pa[32], pb[32];
+#pragma unroll
+      for (int half = 0; half < 2; half++) {
+        uint32_t s0[32], s1[32];
+        tmem_ld32(tl + rA + half * 64, s0);
+        tmem_ld32(tl + rA + half * 64 + 32, s1);
+        tmem_ld_wait(s0);
+        tmem_ld_wait(s1);
+        uint32_t* dst = half ? pb : pa;
+#pragma unroll
+        for (int c = 0; c < 2; c++) {
+#pragma unroll
+          for (int e4 = 0; e4 < 8; e4++) {
+            const float4 l = lse4[half * 16 + c * 8 + e4];
+            const uint32_t* sv = c ? s1 : s0;
+            float pv[4];
+            pv[0] = exp2_approx(fmaf(__uint_as_float(sv[4 * e4 + 0]), sl2, -l.x));
+            pv[1] = exp2_approx(fmaf(__uint_as_float(sv[4 * e4 + 1]), sl2, -l.y));
+            pv[2] = exp2_approx(fmaf(__uint_as_float(sv[4 * e4 + 2]), sl2, -l.z));
+            pv[3] = exp2_approx(fmaf(__uint_as_float(sv[4 * e4 + 3]), sl2, -l.w));
+            if (need_mask) {
+#pragma unroll
+              for (int e = 0; e < 4; e++) {
+                const int q = q0 + half * 64 + c * 32 + 4 * e4 + e;
+                if (q < kv || q >= de) pv[e] = 0.f;
+              }
+            }
+            dst[c * 16 + 2 * e4] = pack_bf16x2(pv[0], pv[1]);
+            dst[c * 16 + 2 * e4 + 1] = pack_bf16x2(pv[2], pv[3]);
+          }
+        }
+      }
+      // P^T over the first 64 columns of region A (their S^T values have been read).
+      tmem_st32(tl + rA, pa);
+      tmem_st32(tl + rA + 32, pb);
+      tmem_st_wait();
+      tc_fence_before();
+      mbar_arrive(&bars->p_full);
+      // dS^T = P^T (dP^T - D), from the bf16 P^T that dV also uses.
+      ok = __all_sync(0xffffffffu, mbar_wait(&bars->dp_full, i & 1, wd));
+      if (!ok) break;
+      tc_fence_after();
+      uint32_t da[32], db[32];
+#pragma unroll
+      for (int half = 0; half < 2; half++) {
+        uint32_t d0[32], d1[32];
+        tmem_ld32(tl + rB + half * 64, d0);
+        tmem_ld32(tl + rB + half * 64 + 32, d1);
+        tmem_ld_wait(d0);
+        tmem_ld_wait(d1);
+        if (half == 1) {  // all of dP^T is in registers: region B may take S^T of the next step
+          tc_fence_before();
+          mbar_arrive(&bars->dp_read);
+        }
+        const uint32_t* src = half ? pb : pa;
+        uint32_t* dst = half ? db : da;
+#pragma unroll
+        for (int c = 0; c < 2; c++) {
+          const uint32_t* dv = c ? d1 : d0;
+#pragma unroll
+          for (int e4 = 0; e4 < 8; e4++) {
+            const float4 dd = del4[half * 16 + c * 8 + e4];
+            const int w = c * 16 + 2 * e4;
+            // bf16 pair -> two floats (first element in the low half)
+            const float p0 = __uint_as_float(src[w] << 16), p1 = __uint_as_float(src[w] & 0xffff0000u);
+            const float p2 = __uint_as_float(src[w + 1] << 16), p3 = __uint_as_float(src[w + 1] & 0xffff0000u);
+            dst[w] = pack_bf16x2(p0 * (__uint_as_float(dv[4 * e4 + 0]) - dd.x),
+                                 p1 * (__uint_as_float(dv[4 * e4 + 1]) - dd.y));
+            dst[w + 1] = pack_bf16x2(p2 * (__uint_as_float(dv[4 * e4 + 2]) - dd.z),
+                                     p3 * (__uint_as_float(dv[4 * e4 + 3]) - dd.w));
+          }
+        }
+      }
+      // dS^T -> this stage's dO buffer, once dP and dV have finished reading dO.
+      ok = __all_sync(0xffffffffu, mbar_wait(&bars->dv_done, i & 1, wd));
+      if (!ok) break;
+      const uint32_t dsb = smem_u32(sDO) + s * C::TILE;
+#pragma unroll
+      for (int c = 0; c < 8; c++) {
+        st_shared_v4(dsb + sw128_offset(r, c), da[4 * c], da[4 * c + 1], da[4 * c + 2], da[4 * c + 3]);
+        st_shared_v4(dsb + C::BLK + sw128_offset(r, c), db[4 * c], db[4 * c + 1], db[4 * c + 2], db[4 * c + 3]);
+      }
+      fence_proxy_async_smem();
+      mbar_arrive(&bars->dss_full);
+    }
+    // Epilogue: dV rows.
+    if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&bars->mma_done, 0, wd));
+    if (ok) {
+      tc_fence_after();
+      __nv_bfloat16* dst = p.dv + ((seq0 + kvc) * p.H + h) * D;
+#pragma unroll 1
+      for (int c = 0; c < D / 32; c++) {
+        uint32_t v[32];
+        tmem_ld32(tl + C::TM_DV + c * 32, v);
+        tmem_ld_wait(v);
+        if (kv < p.L) {
+          uint4* d4 = reinterpret_cast<uint4*>(dst + c * 32);
+#pragma unroll
+          for (int q = 0; q < 4; q++)
+            d4[q] = make_uint4(pack_bf16x2(__uint_as_float(v[8 * q]), __uint_as_float(v[8 * q + 1])),
+                               pack_bf16x2(__uint_as_float(v[8 * q + 2]), __uint_as_float(v[8 * q + 3])),
+                               pack_bf16x2(__uint_as_float(v[8 * q + 4]), __uint_as_float(v[8 * q + 5])),
+                               pack_bf16x2(__uint_as_float(v[8 * q + 6]), __uint_as_float(v[8 * q + 7])));
+        }
+      }
+    }
+  } else {
+    // ---------------- dQ drain warps 4-7: thread t <-> TMEM lane t <-> column d = t of dQ^T
+    const int t = threadIdx.x - 128;
+    const uint32_t tl = tmem + ((uint32_t)((warp - 4) * 32) << 16);
+    bool ok = true;
+    for (int i = 0; i < nq; i++) {
+      ok = __all_sync(0xffffffffu, mbar_wait(&bars->dq_full, i & 1, wd));
+      if (!ok) break;
+      tc_fence_after();
+      const uint32_t rA = C::TM_R + (uint32_t)(i & 1) * 128;
+      uint32_t v[4][32];
+#pragma unroll
+      for (int c = 0; c < 4; c++) tmem_ld32(tl + rA + c * 32, v[c]);
+#pragma unroll
+      for (int c = 0; c < 4; c++) tmem_ld_wait(v[c]);
+      tc_fence_before();
+      mbar_arrive(&bars->r_free);
+      const int q0 = (m_lo + i) * BQ;
+#pragma unroll
+      for (int c = 0; c < 4; c++) {
+        if (t == 0) bulk_wait_read<0>();  // the previous quarter's reduction has read the staging tile
+        named_bar_sync(1, 128);
+#pragma unroll
+        for (int e = 0; e < 32; e++) sSTG[e * D + t] = __uint_as_float(v[c][e]);  // row q = 32c + e, col d = t
+        fence_proxy_async_smem();
+        named_bar_sync(1, 128);
+        if (t == 0) {
+          bulk_reduce_add_f32(p.dq_acc + (vec0 + q0 + 32 * c) * D, sSTG, C::STG_BYTES);
+          bulk_commit();
+        }
+      }
+    }
+    if (t == 0) bulk_wait<0>();
+    // Epilogue: dK rows (scaled).
+    if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&bars->mma_done, 0, wd));
+    if (ok) {
+      tc_fence_after();
+      const int kv = kv0 + t;
+      const int kvc = kv < p.L ? kv : p.L - 1;
+      __nv_bfloat16* dst = p.dk + ((seq0 + kvc) * p.H + h) * D;
+      const float sc = p.scale;
+#pragma unroll 1
+      for (int c = 0; c < D / 32; c++) {
+        uint32_t v[32];
+        tmem_ld32(tl + C::TM_DK + c * 32, v);
+        tmem_ld_wait(v);
+        if (kv < p.L) {
+          uint4* d4 = reinterpret_cast<uint4*>(dst + c * 32);
+#pragma unroll
+          for (int q = 0; q < 4; q++)
+            d4[q] = make_uint4(pack_bf16x2(__uint_as_float(v[8 * q]) * sc, __uint_as_float(v[8 * q + 1]) * sc),
+                               pack_bf16x2(__uint_as_float(v[8 * q + 2]) * sc, __uint_as_float(v[8 * q + 3]) * sc),
+                               pack_bf16x2(__uint_as_float(v[8 * q + 4]) * sc, __uint_as_float(v[8 * q + 5]) * sc),
+                               pack_bf16x2(__uint_as_float(v[8 * q + 6]) * sc, __uint_as_float(v[8 * q + 7]) * sc));
+        }
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 8) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
+cudaError_t launch_attn_bwd_main_d128(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
+                                      const CUtensorMap& tdo, const BwdParams& p, cudaStream_t stream) {
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(attn_bwd_main_d128_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         Bwd128::SMEM_BYTES);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  dim3 grid(p.nkt, p.H, p.B);
+  attn_bwd_main_d128_kernel<<<grid, Bwd128::THREADS, Bwd128::SMEM_BYTES, stream>>>(tq, tk, tv, tdo, p);
+  return cudaGetLastError();
+}
+
+}  // namespace ddattn
