@@ -124,6 +124,15 @@ dd_status dd_attn_clear_status(void* ws, void* stream);
  * (DD_OK, or the first error a kernel recorded there). */
 dd_status dd_attn_poll_status(const void* ws);
 
+/* Self-test of the device-side failure path: launches one warp that waits,
+ * with the same bounded wait the attention kernels use, on an mbarrier that
+ * nothing ever arrives on. After `limit_us` microseconds the wait gives up,
+ * the warp records DD_ERR_DEVICE_TIMEOUT in the status word of `ws` and the
+ * kernel returns normally (no trap, the context stays usable). Returns
+ * DD_ERR_CUDA if the launch fails, else DD_OK; read the outcome with
+ * dd_attn_poll_status. limit_us must be in [1, 1000000]. */
+dd_status dd_selftest_wait_timeout(void* ws, uint32_t limit_us, void* stream);
+
 /* Static description of a status code. */
 const char* dd_status_string(dd_status s);
 

@@ -97,6 +97,22 @@ unsigned long long wait_limit_ns() {
 }
 
 }  // namespace
+
+// One warp waits on an mbarrier that nothing arrives on; the bounded wait
+// expires after limit_ns and records the timeout in *status.
+__global__ void selftest_wait_kernel(int* status, unsigned long long limit_ns) {
+  __shared__ uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x == 0) {
+    abort_flag = 0;
+    mbar_init(&bar, 1);
+    fence_mbar_init();
+  }
+  __syncthreads();
+  Watchdog wd{&abort_flag, status, limit_ns};
+  (void)mbar_wait(&bar, 0, wd);
+}
+
 }  // namespace ddattn
 
 using namespace ddattn;
@@ -186,6 +202,14 @@ dd_status dd_attn_bwd_phases(const dd_attn_desc* desc, const void* q, const void
   p.timeout_ns = wait_limit_ns();
   cudaError_t e = launch_attn_bwd(desc->d, tq, tk, tv, tdo, p, phases, static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? DD_OK : DD_ERR_CUDA;
+}
+
+dd_status dd_selftest_wait_timeout(void* ws, uint32_t limit_us, void* stream) {
+  if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u)) return DD_ERR_WORKSPACE;
+  if (limit_us < 1 || limit_us > 1000000) return DD_ERR_INVALID_ARG;
+  selftest_wait_kernel<<<1, 32, 0, static_cast<cudaStream_t>(stream)>>>(static_cast<int*>(ws),
+                                                                        (unsigned long long)limit_us * 1000ull);
+  return cudaGetLastError() == cudaSuccess ? DD_OK : DD_ERR_CUDA;
 }
 
 dd_status dd_attn_clear_status(void* ws, void* stream) {

@@ -33,7 +33,7 @@ class Desc(ctypes.Structure):
 _lib = None
 
 EXPORTS = ("dd_attn_workspace_size", "dd_attn_fwd", "dd_attn_bwd", "dd_attn_bwd_phases", "dd_attn_bwd_noalloc",
-           "dd_attn_clear_status", "dd_attn_poll_status", "dd_status_string")
+           "dd_attn_clear_status", "dd_attn_poll_status", "dd_selftest_wait_timeout", "dd_status_string")
 NOALLOC_SCRATCH_BYTES = 32 << 20
 DD_BWD_PRE, DD_BWD_MAIN, DD_BWD_POST, DD_BWD_ALL = 1, 2, 4, 7
 
@@ -62,6 +62,8 @@ def lib() -> ctypes.CDLL:
         L.dd_attn_clear_status.restype = i32
         L.dd_attn_poll_status.argtypes = [vp]
         L.dd_attn_poll_status.restype = i32
+        L.dd_selftest_wait_timeout.argtypes = [vp, ctypes.c_uint32, vp]
+        L.dd_selftest_wait_timeout.restype = i32
         L.dd_status_string.argtypes = [i32]
         L.dd_status_string.restype = ctypes.c_char_p
         _lib = L
@@ -149,6 +151,13 @@ def clear_status(workspace, stream=None) -> None:
     st = lib().dd_attn_clear_status(workspace.data_ptr(), _stream(stream))
     if st != DD_OK:
         raise DDAttnError(st, "dd_attn_clear_status")
+
+
+def selftest_wait_timeout(workspace, limit_us: int = 20000, stream=None) -> None:
+    """Launch the bounded-wait self-test kernel (see dd_selftest_wait_timeout)."""
+    st = lib().dd_selftest_wait_timeout(workspace.data_ptr(), int(limit_us), _stream(stream))
+    if st != DD_OK:
+        raise DDAttnError(st, "dd_selftest_wait_timeout")
 
 
 def poll_status(workspace) -> int:
