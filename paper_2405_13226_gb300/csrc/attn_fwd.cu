@@ -6,34 +6,34 @@
 // the first row's document start). Warp roles:
 //   warps 0-3  softmax: thread r owns query row r = TMEM lane r. Reads the
 //              S tile from TMEM, masks (diagonal / document-edge tiles only),
-//              online max/sum in the log2 domain, writes P (bf16) to a
-//              128B-swizzled smem tile, and rescales O in TMEM when the
-//              running max grows by more than 2^8 (otherwise the stale max
-//              is kept; P <= 256 stays exact enough in bf16/fp32).
-//   warp 4     TMA producer for Q (once) and K tiles (2-stage ring); TMEM alloc.
-//   warp 5     TMA producer for V tiles (2-stage ring).
+//              online max/sum in the log2 domain, writes P (bf16 pairs) back
+//              over the first 64 columns of the same TMEM buffer, and
+//              rescales O in TMEM when the running max grows by more than 2^8
+//              (otherwise the stale max is kept; P <= 256 stays exact enough
+//              in bf16/fp32).
+//   warp 4     TMA producer for Q (once) and K tiles (3-stage ring); TMEM alloc.
+//   warp 5     TMA producer for V tiles (3-stage ring).
 //   warp 6     one thread issues tcgen05.mma: S[j%2] = Q K_j^T (TMEM, fp32),
-//              then O += P_{j-1} V_{j-1} (TMEM, fp32), so the tensor core
-//              computes S_{j+1} while the softmax warps work on S_j.
+//              then O += P_{j-1} V_{j-1} with P read from TMEM (the .ts form),
+//              so the tensor core computes S_{j+1} while the softmax warps
+//              work on S_j.
+// TMEM: S buffers at columns 0 and 128 (P over their first 64 columns), O at 256.
 #include "common.cuh"
 
 namespace ddattn {
 
 template <int D>
 struct FwdCfg {
-  static constexpr int BM = 128, BN = 128;
+  static constexpr int BM = 128, BN = 128, STAGES = 3;
   static constexpr int DB = D / 64;                    // 64-column swizzle blocks per row
   static constexpr int Q_BLK = BM * 128;               // bytes of one [128 rows][64] block
   static constexpr int KV_BLK = BN * 128;
   static constexpr int Q_BYTES = DB * Q_BLK;
   static constexpr int KV_BYTES = DB * KV_BLK;
-  static constexpr int P_BLK = BM * 128;
-  static constexpr int P_BYTES = 2 * P_BLK;            // [128 q][128 kv] bf16
   static constexpr int OFF_Q = 0;
   static constexpr int OFF_K = OFF_Q + Q_BYTES;
-  static constexpr int OFF_V = OFF_K + 2 * KV_BYTES;
-  static constexpr int OFF_P = OFF_V + 2 * KV_BYTES;
-  static constexpr int OFF_BAR = OFF_P + 2 * P_BYTES;
+  static constexpr int OFF_V = OFF_K + STAGES * KV_BYTES;
+  static constexpr int OFF_BAR = OFF_V + STAGES * KV_BYTES;
   static constexpr int SMEM_BYTES = OFF_BAR + 256 + 1024;
   static constexpr uint32_t TMEM_S = 0;                // S buffers at columns 0 and 128
   static constexpr uint32_t TMEM_O = 256;              // O: D columns
@@ -43,8 +43,8 @@ struct FwdCfg {
 
 struct FwdBars {
   uint64_t q_full;
-  uint64_t k_full[2], k_empty[2], v_full[2], v_empty[2];
-  uint64_t s_full[2], s_free[2], p_full[2], p_empty[2];
+  uint64_t k_full[3], k_empty[3], v_full[3], v_empty[3];
+  uint64_t s_full[2], p_full[2], pv_done[2];
   uint64_t mma_drain;
   uint32_t tmem_base;
   int abort_flag;
@@ -56,6 +56,7 @@ __global__ void __launch_bounds__(224, 1)
     attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                     const __grid_constant__ CUtensorMap tmV, const FwdParams p) {
   using C = FwdCfg<D>;
+  constexpr int ST = C::STAGES;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
   FwdBars* bars = reinterpret_cast<FwdBars*>(smem + C::OFF_BAR);
@@ -75,15 +76,16 @@ __global__ void __launch_bounds__(224, 1)
   if (threadIdx.x == 0) {
     bars->abort_flag = 0;
     mbar_init(&bars->q_full, 1);
-    for (int i = 0; i < 2; i++) {
+    for (int i = 0; i < ST; i++) {
       mbar_init(&bars->k_full[i], 1);
       mbar_init(&bars->k_empty[i], 1);
       mbar_init(&bars->v_full[i], 1);
       mbar_init(&bars->v_empty[i], 1);
+    }
+    for (int i = 0; i < 2; i++) {
       mbar_init(&bars->s_full[i], 1);
-      mbar_init(&bars->s_free[i], 128);
       mbar_init(&bars->p_full[i], 128);
-      mbar_init(&bars->p_empty[i], 1);
+      mbar_init(&bars->pv_done[i], 1);
     }
     mbar_init(&bars->mma_drain, 1);
     fence_mbar_init();
@@ -99,7 +101,6 @@ __global__ void __launch_bounds__(224, 1)
   uint8_t* sQ = smem + C::OFF_Q;
   uint8_t* sK = smem + C::OFF_K;
   uint8_t* sV = smem + C::OFF_V;
-  uint8_t* sP = smem + C::OFF_P;
 
   if (warp == 4) {
     // ---------------- Q + K producer
@@ -110,8 +111,8 @@ __global__ void __launch_bounds__(224, 1)
       for (int blk = 0; blk < C::DB; blk++) tma_load_4d(sQ + blk * C::Q_BLK, &tmQ, &bars->q_full, 64 * blk, h, row0, b);
       int issued = 0;
       for (int j = 0; j < nt; j++) {
-        const int s = j & 1;
-        if (j >= 2 && !mbar_wait(&bars->k_empty[s], ((j >> 1) - 1) & 1, wd)) break;
+        const int s = j % ST;
+        if (j >= ST && !mbar_wait(&bars->k_empty[s], ((j / ST) - 1) & 1, wd)) break;
         mbar_arrive_expect_tx(&bars->k_full[s], C::KV_BYTES);
         const int kv0 = (n_lo + j) * C::BN;
         for (int blk = 0; blk < C::DB; blk++)
@@ -120,8 +121,8 @@ __global__ void __launch_bounds__(224, 1)
       }
       if (*wd.abort_flag) {  // let in-flight copies land before the CTA exits
         mbar_wait_drain(&bars->q_full, 0, wd.limit_ns);
-        for (int j = issued - 2 < 0 ? 0 : issued - 2; j < issued; j++)
-          mbar_wait_drain(&bars->k_full[j & 1], (j >> 1) & 1, wd.limit_ns);
+        for (int j = issued - ST < 0 ? 0 : issued - ST; j < issued; j++)
+          mbar_wait_drain(&bars->k_full[j % ST], (j / ST) & 1, wd.limit_ns);
       }
     }
   } else if (warp == 5) {
@@ -130,8 +131,8 @@ __global__ void __launch_bounds__(224, 1)
       prefetch_tmap(&tmV);
       int issued = 0;
       for (int j = 0; j < nt; j++) {
-        const int s = j & 1;
-        if (j >= 2 && !mbar_wait(&bars->v_empty[s], ((j >> 1) - 1) & 1, wd)) break;
+        const int s = j % ST;
+        if (j >= ST && !mbar_wait(&bars->v_empty[s], ((j / ST) - 1) & 1, wd)) break;
         mbar_arrive_expect_tx(&bars->v_full[s], C::KV_BYTES);
         const int kv0 = (n_lo + j) * C::BN;
         for (int blk = 0; blk < C::DB; blk++)
@@ -139,44 +140,46 @@ __global__ void __launch_bounds__(224, 1)
         issued = j + 1;
       }
       if (*wd.abort_flag)
-        for (int j = issued - 2 < 0 ? 0 : issued - 2; j < issued; j++)
-          mbar_wait_drain(&bars->v_full[j & 1], (j >> 1) & 1, wd.limit_ns);
+        for (int j = issued - ST < 0 ? 0 : issued - ST; j < issued; j++)
+          mbar_wait_drain(&bars->v_full[j % ST], (j / ST) & 1, wd.limit_ns);
     }
   } else if (warp == 6) {
     // ---------------- MMA issuer
     if (lane == 0) {
       constexpr uint32_t idesc_s = idesc_bf16(128, 128, false, false);  // Q, K both K-major
-      constexpr uint32_t idesc_o = idesc_bf16(128, D, false, true);      // P K-major, V MN-major
-      const uint32_t aQ = smem_u32(sQ), aK = smem_u32(sK), aV = smem_u32(sV), aP = smem_u32(sP);
+      constexpr uint32_t idesc_o = idesc_bf16(128, D, false, true);      // P (TMEM) x V (MN-major)
+      const uint32_t aQ = smem_u32(sQ), aK = smem_u32(sK), aV = smem_u32(sV);
       if (mbar_wait(&bars->q_full, 0, wd)) {
         for (int j = 0; j <= nt; j++) {
           if (j < nt) {
-            const int s = j & 1;
-            if (!mbar_wait(&bars->k_full[s], (j >> 1) & 1, wd)) break;
-            if (j >= 2 && !mbar_wait(&bars->s_free[s], ((j >> 1) - 1) & 1, wd)) break;
+            const int ks = j % ST, sb = j & 1;
+            if (!mbar_wait(&bars->k_full[ks], (j / ST) & 1, wd)) break;
+            // S[sb] holds P_{j-2} until PV_{j-2} has read it.
+            if (j >= 2 && !mbar_wait(&bars->pv_done[sb], ((j >> 1) - 1) & 1, wd)) break;
             tc_fence_after();
 #pragma unroll
-            for (int ks = 0; ks < D / 16; ks++) {
-              const uint64_t da = sdesc_sw128(aQ + (ks >> 2) * C::Q_BLK + (ks & 3) * 32, 16, 1024);
-              const uint64_t db = sdesc_sw128(aK + s * C::KV_BYTES + (ks >> 2) * C::KV_BLK + (ks & 3) * 32, 16, 1024);
-              umma_bf16(tmem + C::TMEM_S + s * 128, da, db, idesc_s, ks > 0 ? 1u : 0u);
+            for (int kk = 0; kk < D / 16; kk++) {
+              const uint64_t da = sdesc_sw128(aQ + (kk >> 2) * C::Q_BLK + (kk & 3) * 32, 16, 1024);
+              const uint64_t db =
+                  sdesc_sw128(aK + ks * C::KV_BYTES + (kk >> 2) * C::KV_BLK + (kk & 3) * 32, 16, 1024);
+              umma_bf16(tmem + C::TMEM_S + sb * 128, da, db, idesc_s, kk > 0 ? 1u : 0u);
             }
-            umma_commit(&bars->s_full[s]);
-            umma_commit(&bars->k_empty[s]);
+            umma_commit(&bars->s_full[sb]);
+            umma_commit(&bars->k_empty[ks]);
           }
           if (j >= 1) {
-            const int i = j - 1, s = i & 1;
-            if (!mbar_wait(&bars->v_full[s], (i >> 1) & 1, wd)) break;
-            if (!mbar_wait(&bars->p_full[s], (i >> 1) & 1, wd)) break;
+            const int i = j - 1, vs = i % ST, pb = i & 1;
+            if (!mbar_wait(&bars->v_full[vs], (i / ST) & 1, wd)) break;
+            if (!mbar_wait(&bars->p_full[pb], (i >> 1) & 1, wd)) break;
             tc_fence_after();
 #pragma unroll
-            for (int ks = 0; ks < C::BN / 16; ks++) {
-              const uint64_t da = sdesc_sw128(aP + s * C::P_BYTES + (ks >> 2) * C::P_BLK + (ks & 3) * 32, 16, 1024);
-              const uint64_t db = sdesc_sw128(aV + s * C::KV_BYTES + ks * 2048, C::KV_BLK, 1024);
-              umma_bf16(tmem + C::TMEM_O, da, db, idesc_o, (i > 0 || ks > 0) ? 1u : 0u);
+            for (int kk = 0; kk < C::BN / 16; kk++) {
+              const uint64_t db = sdesc_sw128(aV + vs * C::KV_BYTES + kk * 2048, C::KV_BLK, 1024);
+              umma_bf16_ts(tmem + C::TMEM_O, tmem + C::TMEM_S + pb * 128 + kk * 8, db, idesc_o,
+                           (i > 0 || kk > 0) ? 1u : 0u);
             }
-            umma_commit(&bars->p_empty[s]);
-            umma_commit(&bars->v_empty[s]);
+            umma_commit(&bars->pv_done[pb]);
+            umma_commit(&bars->v_empty[vs]);
           }
         }
       }
@@ -191,25 +194,25 @@ __global__ void __launch_bounds__(224, 1)
     const int ds = (int)(doc_start(p.offsets, p.n_offsets, seq0 + rowc, seq0) - seq0);
     const uint32_t tl = tmem + ((uint32_t)(warp * 32) << 16);
     const float sl2 = p.scale_log2;
+    const uint64_t sl2x2 = f32x2(sl2, sl2);
     float m_run = -INFINITY, l_run = 0.f;
     bool ok = true;
     for (int j = 0; j < nt && ok; j++) {
-      const int s = j & 1;
+      const int sb = j & 1;
       const int kv0 = (n_lo + j) * C::BN;
-      ok = __all_sync(0xffffffffu, mbar_wait(&bars->s_full[s], (j >> 1) & 1, wd));
+      const uint32_t sbuf = tl + C::TMEM_S + sb * 128;
+      ok = __all_sync(0xffffffffu, mbar_wait(&bars->s_full[sb], (j >> 1) & 1, wd));
       if (!ok) break;
       tc_fence_after();
       uint32_t v0[32], v1[32], v2[32], v3[32];
-      tmem_ld32(tl + C::TMEM_S + s * 128 + 0, v0);
-      tmem_ld32(tl + C::TMEM_S + s * 128 + 32, v1);
-      tmem_ld32(tl + C::TMEM_S + s * 128 + 64, v2);
-      tmem_ld32(tl + C::TMEM_S + s * 128 + 96, v3);
+      tmem_ld32(sbuf + 0, v0);
+      tmem_ld32(sbuf + 32, v1);
+      tmem_ld32(sbuf + 64, v2);
+      tmem_ld32(sbuf + 96, v3);
       tmem_ld_wait(v0);
       tmem_ld_wait(v1);
       tmem_ld_wait(v2);
       tmem_ld_wait(v3);
-      tc_fence_before();
-      mbar_arrive(&bars->s_free[s]);
       float sc[128];
 #pragma unroll
       for (int c = 0; c < 32; c++) {
@@ -237,31 +240,25 @@ __global__ void __launch_bounds__(224, 1)
         m_run = m_tile;
       }
       const float m_use = (m_run == -INFINITY) ? 0.f : m_run;
-      float rs = 0.f;
-      uint32_t pk[64];
+      const uint64_t negm = f32x2(-m_use, -m_use);
+      uint64_t rs2 = f32x2(0.f, 0.f);
+      uint32_t pk0[32], pk1[32];
 #pragma unroll
       for (int c = 0; c < 64; c++) {
-        const float p0 = exp2_approx(fmaf(sc[2 * c], sl2, -m_use));
-        const float p1 = exp2_approx(fmaf(sc[2 * c + 1], sl2, -m_use));
-        rs += p0 + p1;
-        pk[c] = pack_bf16x2(p0, p1);
+        const uint64_t x = fma_f32x2(f32x2(sc[2 * c], sc[2 * c + 1]), sl2x2, negm);
+        const float p0 = exp2_approx(f32x2_lo(x));
+        const float p1 = exp2_approx(f32x2_hi(x));
+        rs2 = add_f32x2(rs2, f32x2(p0, p1));
+        if (c < 32) pk0[c] = pack_bf16x2(p0, p1);
+        else pk1[c - 32] = pack_bf16x2(p0, p1);
       }
-      l_run = l_run * alpha + rs;
-      // P_j -> smem buffer j%2 (free once PV_{j-2} completed)
-      if (j >= 2) {
-        ok = __all_sync(0xffffffffu, mbar_wait(&bars->p_empty[s], ((j >> 1) - 1) & 1, wd));
-        if (!ok) break;
-      }
-      const uint32_t pbase = smem_u32(sP) + s * C::P_BYTES;
-#pragma unroll
-      for (int c = 0; c < 16; c++) {
-        const uint32_t addr = pbase + (c >> 3) * C::P_BLK + sw128_offset(r, c & 7);
-        st_shared_v4(addr, pk[4 * c], pk[4 * c + 1], pk[4 * c + 2], pk[4 * c + 3]);
-      }
-      fence_proxy_async_smem();
+      l_run = l_run * alpha + (f32x2_lo(rs2) + f32x2_hi(rs2));
+      // P_j over the first 64 columns of its S buffer (all of S_j has been read).
+      tmem_st32(sbuf + 0, pk0);
+      tmem_st32(sbuf + 32, pk1);
       // O *= alpha, after PV_{j-1} landed and before PV_j is issued.
       if (__any_sync(0xffffffffu, rescale)) {
-        ok = __all_sync(0xffffffffu, mbar_wait(&bars->p_empty[(j - 1) & 1], ((j - 1) >> 1) & 1, wd));
+        ok = __all_sync(0xffffffffu, mbar_wait(&bars->pv_done[(j - 1) & 1], ((j - 1) >> 1) & 1, wd));
         if (!ok) break;
         tc_fence_after();
 #pragma unroll 1
@@ -273,13 +270,13 @@ __global__ void __launch_bounds__(224, 1)
           for (int e = 0; e < 32; e++) ov[e] = __float_as_uint(__uint_as_float(ov[e]) * alpha);
           tmem_st32(tl + C::TMEM_O + c * 32, ov);
         }
-        tmem_st_wait();
       }
+      tmem_st_wait();
       tc_fence_before();
-      mbar_arrive(&bars->p_full[s]);
+      mbar_arrive(&bars->p_full[sb]);
     }
     // Epilogue: O / l -> bf16, LSE = (m + log2 l) * ln2.
-    if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&bars->p_empty[(nt - 1) & 1], ((nt - 1) >> 1) & 1, wd));
+    if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&bars->pv_done[(nt - 1) & 1], ((nt - 1) >> 1) & 1, wd));
     if (ok) {
       tc_fence_after();
       const float inv_l = l_run > 0.f ? 1.f / l_run : 0.f;
