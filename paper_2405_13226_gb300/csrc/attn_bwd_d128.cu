@@ -12,8 +12,9 @@
 //
 // TMEM (512 columns): two 128-column regions R[0], R[1] whose roles alternate
 // every step (A = R[i % 2], B = R[(i + 1) % 2]):
-//   A: S^T (fp32) -> P^T (bf16 pairs over its first 64 columns, A operand of
-//      dV) -> dQ^T (fp32, after dV has read P^T) -> dP^T of step i + 1
+//   A: S^T (fp32) -> P^T (bf16 pairs: queries 0-63 over columns 0-31, queries
+//      64-127 over columns 64-95, the A operand of dV) -> dQ^T (fp32, after dV
+//      has read P^T) -> dP^T of step i + 1
 //   B: dP^T (fp32) -> S^T of step i + 1 (as soon as dP^T is in registers)
 //   dV [256,384), dK [384,512) accumulate over the steps.
 // The tensor core runs dV_i, S_{i+1}, dK_i, dQ^T_i, dP_{i+1}, dV_{i+1}, ... so
@@ -27,9 +28,13 @@
 // contiguous accumulator rows (a direct red.global per element was measured
 // slower: its load/store traffic delays the P/dS warps on the same SM).
 //
-// Warp roles: 0-3 P/dS (thread r <-> key row r <-> TMEM lane r) and the dV
-// epilogue; 4-7 dQ drain and the dK epilogue; 8 TMA producer (and TMEM owner);
-// 9 issues tcgen05.mma.
+// Warp roles, one warpgroup each (thread r of a group <-> key row r <-> TMEM
+// lane r): WG0 / WG1 compute P and dS for query columns 0-63 / 64-127 and write
+// the matching half of dV; WG2 drains dQ and writes dK; WG3: warp 12 is the TMA
+// producer and TMEM owner, warp 13 issues tcgen05.mma. The block launches with
+// 128 registers per thread; WG3 gives registers back (setmaxnreg.dec to 56) and
+// the other three groups take them (setmaxnreg.inc to 152): 4*32*56 +
+// 12*32*152 = 65536, exactly the launch's register file share.
 #include "common.cuh"
 
 namespace ddattn {
@@ -49,8 +54,10 @@ struct Bwd128 {
   static constexpr int OFF_BAR = OFF_DEL + 2 * BQ * 4;
   static constexpr int SMEM_BYTES = OFF_BAR + 256 + 1024;
   static constexpr uint32_t TM_R = 0, TM_DV = 256, TM_DK = 384;  // R[k] at TM_R + 128 k
-  static constexpr int THREADS = 320;
+  static constexpr int THREADS = 512;
+  static constexpr int REGS_LOW = 56, REGS_HIGH = 152;   // setmaxnreg split, see above
 };
+static_assert(4 * 32 * Bwd128::REGS_LOW + 12 * 32 * Bwd128::REGS_HIGH == 512 * 128, "register split");
 
 struct Bwd128Bars {
   uint64_t kv_full;
@@ -62,7 +69,16 @@ struct Bwd128Bars {
 };
 static_assert(sizeof(Bwd128Bars) <= 256, "barrier block");
 
-__global__ void __launch_bounds__(320, 1)
+template <uint32_t N>
+__device__ __forceinline__ void setmaxnreg_inc() {
+  asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(N));
+}
+template <uint32_t N>
+__device__ __forceinline__ void setmaxnreg_dec() {
+  asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(N));
+}
+
+__global__ void __launch_bounds__(512, 1)
     attn_bwd_main_d128_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                               const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmDO,
                               const BwdParams p) {
@@ -93,16 +109,16 @@ __global__ void __launch_bounds__(320, 1)
     }
     mbar_init(&bars->s_full, 1);
     mbar_init(&bars->dp_full, 1);
-    mbar_init(&bars->p_full, 128);
-    mbar_init(&bars->dp_read, 128);
-    mbar_init(&bars->dss_full, 128);
+    mbar_init(&bars->p_full, 256);
+    mbar_init(&bars->dp_read, 256);
+    mbar_init(&bars->dss_full, 256);
     mbar_init(&bars->dv_done, 1);
     mbar_init(&bars->dq_full, 1);
     mbar_init(&bars->r_free, 128);
     mbar_init(&bars->mma_done, 1);
     fence_mbar_init();
   }
-  if (warp == 8) {
+  if (warp == 12) {
     tmem_alloc(&bars->tmem_base, 512);
     tmem_relinquish();
   }
@@ -119,7 +135,10 @@ __global__ void __launch_bounds__(320, 1)
   float* sDEL = reinterpret_cast<float*>(smem + C::OFF_DEL);
   const long long vec0 = ((long long)b * p.H + h) * p.L128;  // row 0 of this (b, h) in the padded vectors
 
-  if (warp == 8) {
+  const int wg = warp >> 2;
+  if (wg == 3) {
+  setmaxnreg_dec<C::REGS_LOW>();
+  if (warp == 12) {
     // ---------------- TMA producer
     if (lane == 0) {
       prefetch_tmap(&tmQ);
@@ -151,49 +170,53 @@ __global__ void __launch_bounds__(320, 1)
           mbar_wait_drain(&bars->q_full[i & 1], (i >> 1) & 1, wd.limit_ns);
       }
     }
-  } else if (warp == 9) {
+  } else if (warp == 13) {
     // ---------------- MMA issuer
     if (lane == 0) {
       constexpr uint32_t id_s = idesc_bf16(128, 128, false, false);  // K / V rows x Q / dO rows (K-major)
       constexpr uint32_t id_kv = idesc_bf16(128, 128, false, true);  // P^T (TMEM) / dS^T (smem) x dO / Q (MN-major)
       constexpr uint32_t id_dq = idesc_bf16(128, 128, true, true);   // K^T (MN-major) x dS^T (MN-major)
-      const uint32_t aK = smem_u32(sK), aV = smem_u32(sV), aQ = smem_u32(sQ), aDO = smem_u32(sDO);
+      // Descriptors are built once and advanced by adding (byte offset >> 4) to the
+      // 14-bit start-address field (all smem offsets here stay below 256 KB).
+      const uint64_t dK_k0 = sdesc_sw128(smem_u32(sK), 16, 1024);          // K-major views
+      const uint64_t dV_k0 = sdesc_sw128(smem_u32(sV), 16, 1024);
+      const uint64_t dQ_k0 = sdesc_sw128(smem_u32(sQ), 16, 1024);
+      const uint64_t dO_k0 = sdesc_sw128(smem_u32(sDO), 16, 1024);
+      const uint64_t dK_mn0 = sdesc_sw128(smem_u32(sK), C::BLK, 1024);     // MN-major views
+      const uint64_t dQ_mn0 = sdesc_sw128(smem_u32(sQ), C::BLK, 1024);
+      const uint64_t dO_mn0 = sdesc_sw128(smem_u32(sDO), C::BLK, 1024);
       bool ok = mbar_wait(&bars->kv_full, 0, wd) && mbar_wait(&bars->q_full[0], 0, wd);
-      auto issue_s = [&](int j, uint32_t reg) {  // S^T_j = K Q_j^T into region `reg`
-        const uint32_t qs = aQ + (j & 1) * C::TILE;
-#pragma unroll
-        for (int ks = 0; ks < 8; ks++) {
-          const uint32_t off = (ks >> 2) * C::BLK + (ks & 3) * 32;
-          umma_bf16(tmem + reg, sdesc_sw128(aK + off, 16, 1024), sdesc_sw128(qs + off, 16, 1024), id_s,
-                    ks > 0 ? 1u : 0u);
-        }
-        umma_commit(&bars->s_full);
-      };
-      auto issue_dp = [&](int j, uint32_t reg) {  // dP^T_j = V dO_j^T into region `reg`
-        const uint32_t os = aDO + (j & 1) * C::TILE;
-#pragma unroll
-        for (int ks = 0; ks < 8; ks++) {
-          const uint32_t off = (ks >> 2) * C::BLK + (ks & 3) * 32;
-          umma_bf16(tmem + reg, sdesc_sw128(aV + off, 16, 1024), sdesc_sw128(os + off, 16, 1024), id_s,
-                    ks > 0 ? 1u : 0u);
-        }
-        umma_commit(&bars->dp_full);
-      };
       if (ok) {
         tc_fence_after();
-        issue_s(0, C::TM_R);
-        issue_dp(0, C::TM_R + 128);
+#pragma unroll
+        for (int ks = 0; ks < 8; ks++) {  // S^T_0 = K Q_0^T into R[0]
+          const uint32_t off = ((ks >> 2) * C::BLK + (ks & 3) * 32) >> 4;
+          umma_bf16(tmem + C::TM_R, dK_k0 + off, dQ_k0 + off, id_s, ks > 0 ? 1u : 0u);
+        }
+        umma_commit(&bars->s_full);
+#pragma unroll
+        for (int ks = 0; ks < 8; ks++) {  // dP^T_0 = V dO_0^T into R[1]
+          const uint32_t off = ((ks >> 2) * C::BLK + (ks & 3) * 32) >> 4;
+          umma_bf16(tmem + C::TM_R + 128, dV_k0 + off, dO_k0 + off, id_s, ks > 0 ? 1u : 0u);
+        }
+        umma_commit(&bars->dp_full);
       }
       for (int i = 0; ok && i < nq; i++) {
         const int s = i & 1;
         const uint32_t rA = C::TM_R + (uint32_t)(i & 1) * 128, rB = C::TM_R + (uint32_t)((i + 1) & 1) * 128;
-        const uint32_t qs = aQ + s * C::TILE, os = aDO + s * C::TILE;
+        const uint32_t st = (uint32_t)(s * C::TILE) >> 4, st1 = (uint32_t)(((i + 1) & 1) * C::TILE) >> 4;
+        // Opaque copies of the base descriptors: keeps the 40 derived
+        // descriptors of a step from being hoisted out of the loop (which would
+        // hold them all in registers at once).
+        const uint64_t dK_k = opaque_u64(dK_k0), dV_k = opaque_u64(dV_k0), dQ_k = opaque_u64(dQ_k0),
+                       dO_k = opaque_u64(dO_k0), dK_mn = opaque_u64(dK_mn0), dQ_mn = opaque_u64(dQ_mn0),
+                       dO_mn = opaque_u64(dO_mn0);
         // dV += P^T dO  (A: P^T in region A, 8 columns per 16 queries)
         if (!(ok = mbar_wait(&bars->p_full, i & 1, wd))) break;
         tc_fence_after();
 #pragma unroll
-        for (int ks = 0; ks < 8; ks++)
-          umma_bf16_ts(tmem + C::TM_DV, tmem + rA + ks * 8, sdesc_sw128(os + ks * 2048, C::BLK, 1024), id_kv,
+        for (int ks = 0; ks < 8; ks++)  // queries 16 ks..: columns 8 ks (+32 for the second group's half)
+          umma_bf16_ts(tmem + C::TM_DV, tmem + rA + ks * 8 + (ks >= 4 ? 32 : 0), dO_mn + st + ks * (2048 >> 4), id_kv,
                        (i > 0 || ks > 0) ? 1u : 0u);
         umma_commit(&bars->dv_done);
         // S^T_{i+1} into region B as soon as dP^T_i has been read out of it.
@@ -202,43 +225,55 @@ __global__ void __launch_bounds__(320, 1)
                      mbar_wait(&bars->dp_read, i & 1, wd)))
             break;
           tc_fence_after();
-          issue_s(i + 1, rB);
+#pragma unroll
+          for (int ks = 0; ks < 8; ks++) {
+            const uint32_t off = ((ks >> 2) * C::BLK + (ks & 3) * 32) >> 4;
+            umma_bf16(tmem + rB, dK_k + off, dQ_k + st1 + off, id_s, ks > 0 ? 1u : 0u);
+          }
+          umma_commit(&bars->s_full);
         }
         // dK += dS^T Q  (A: dS^T in this stage's dO buffer, K-major view)
         if (!(ok = mbar_wait(&bars->dss_full, i & 1, wd))) break;
         tc_fence_after();
 #pragma unroll
         for (int ks = 0; ks < 8; ks++) {
-          const uint32_t off = (ks >> 2) * C::BLK + (ks & 3) * 32;
-          umma_bf16(tmem + C::TM_DK, sdesc_sw128(os + off, 16, 1024), sdesc_sw128(qs + ks * 2048, C::BLK, 1024),
-                    id_kv, (i > 0 || ks > 0) ? 1u : 0u);
+          const uint32_t off = ((ks >> 2) * C::BLK + (ks & 3) * 32) >> 4;
+          umma_bf16(tmem + C::TM_DK, dO_k + st + off, dQ_mn + st + ks * (2048 >> 4), id_kv,
+                    (i > 0 || ks > 0) ? 1u : 0u);
         }
         // dQ^T = K^T dS^T into region A (dV_i has finished reading P^T there:
         // dss_full is only raised after dv_done).
-        tc_fence_after();
 #pragma unroll
         for (int ks = 0; ks < 8; ks++)
-          umma_bf16(tmem + rA, sdesc_sw128(aK + ks * 2048, C::BLK, 1024), sdesc_sw128(os + ks * 2048, C::BLK, 1024),
-                    id_dq, ks > 0 ? 1u : 0u);
+          umma_bf16(tmem + rA, dK_mn + ks * (2048 >> 4), dO_mn + st + ks * (2048 >> 4), id_dq, ks > 0 ? 1u : 0u);
         umma_commit(&bars->dq_full);
         umma_commit(&bars->q_empty[s]);
         // dP^T_{i+1} into region A once the drain has read dQ^T_i out of it.
         if (i + 1 < nq) {
           if (!(ok = mbar_wait(&bars->r_free, i & 1, wd))) break;
           tc_fence_after();
-          issue_dp(i + 1, rA);
+#pragma unroll
+          for (int ks = 0; ks < 8; ks++) {
+            const uint32_t off = ((ks >> 2) * C::BLK + (ks & 3) * 32) >> 4;
+            umma_bf16(tmem + rA, dV_k + off, dO_k + st1 + off, id_s, ks > 0 ? 1u : 0u);
+          }
+          umma_commit(&bars->dp_full);
         }
       }
       umma_commit(&bars->mma_done);
       mbar_wait_drain(&bars->mma_done, 0, wd.limit_ns);
     }
-  } else if (warp < 4) {
-    // ---------------- P / dS warps
-    const int r = threadIdx.x;
+  }
+  } else {
+  setmaxnreg_inc<C::REGS_HIGH>();
+  if (wg < 2) {
+    // ---------------- P / dS warps: group wg handles query columns [64 wg, 64 wg + 64)
+    const int r = threadIdx.x & 127;
+    const int qh = wg * 64;
     const int kv = kv0 + r;
     const int kvc = kv < p.L ? kv : p.L - 1;
     const int de = (int)(doc_end(p.offsets, p.n_offsets, seq0 + kvc, seq0 + p.L) - seq0);
-    const uint32_t tl = tmem + ((uint32_t)(warp * 32) << 16);
+    const uint32_t tl = tmem + ((uint32_t)((warp & 3) * 32) << 16);
     const float sl2 = p.scale_log2;
     bool ok = true;
     for (int i = 0; i < nq && ok; i++) {
@@ -249,24 +284,22 @@ __global__ void __launch_bounds__(320, 1)
                       mbar_wait(&bars->s_full, i & 1, wd) && mbar_wait(&bars->q_full[s], (i >> 1) & 1, wd));
       if (!ok) break;
       tc_fence_after();
-      const float4* lse4 = reinterpret_cast<const float4*>(sLSE + s * BQ);
-      const float4* del4 = reinterpret_cast<const float4*>(sDEL + s * BQ);
-      const bool need_mask = (q0 < kv) || (q0 + BQ > de);
-      // P^T packed as bf16 pairs: pa = queries 0..63, pb = queries 64..127.
-      uint32_t pa[32], pb[32];
-#pragma unroll
-      for (int half = 0; half < 2; half++) {
+      const float4* lse4 = reinterpret_cast<const float4*>(sLSE + s * BQ + qh);
+      const float4* del4 = reinterpret_cast<const float4*>(sDEL + s * BQ + qh);
+      const bool need_mask = (q0 + qh < kv) || (q0 + qh + 64 > de);
+      // P^T of this group's 64 query columns, packed as bf16 pairs.
+      uint32_t pk[32];
+      {
         uint32_t s0[32], s1[32];
-        tmem_ld32(tl + rA + half * 64, s0);
-        tmem_ld32(tl + rA + half * 64 + 32, s1);
+        tmem_ld32(tl + rA + qh, s0);
+        tmem_ld32(tl + rA + qh + 32, s1);
         tmem_ld_wait(s0);
         tmem_ld_wait(s1);
-        uint32_t* dst = half ? pb : pa;
 #pragma unroll
         for (int c = 0; c < 2; c++) {
 #pragma unroll
           for (int e4 = 0; e4 < 8; e4++) {
-            const float4 l = lse4[half * 16 + c * 8 + e4];
+            const float4 l = lse4[c * 8 + e4];
             const uint32_t* sv = c ? s1 : s0;
             float pv[4];
             pv[0] = exp2_approx(fmaf(__uint_as_float(sv[4 * e4 + 0]), sl2, -l.x));
@@ -276,18 +309,18 @@ __global__ void __launch_bounds__(320, 1)
             if (need_mask) {
 #pragma unroll
               for (int e = 0; e < 4; e++) {
-                const int q = q0 + half * 64 + c * 32 + 4 * e4 + e;
+                const int q = q0 + qh + c * 32 + 4 * e4 + e;
                 if (q < kv || q >= de) pv[e] = 0.f;
               }
             }
-            dst[c * 16 + 2 * e4] = pack_bf16x2(pv[0], pv[1]);
-            dst[c * 16 + 2 * e4 + 1] = pack_bf16x2(pv[2], pv[3]);
+            pk[c * 16 + 2 * e4] = pack_bf16x2(pv[0], pv[1]);
+            pk[c * 16 + 2 * e4 + 1] = pack_bf16x2(pv[2], pv[3]);
           }
         }
       }
-      // P^T over the first 64 columns of region A (their S^T values have been read).
-      tmem_st32(tl + rA, pa);
-      tmem_st32(tl + rA + 32, pb);
+      // P^T over the first 32 of this group's own 64 S^T columns of region A
+      // (queries 64 wg .. 64 wg + 63 as bf16 pairs; this group has read them).
+      tmem_st32(tl + rA + wg * 64, pk);
       tmem_st_wait();
       tc_fence_before();
       mbar_arrive(&bars->p_full);
@@ -295,46 +328,39 @@ __global__ void __launch_bounds__(320, 1)
       ok = __all_sync(0xffffffffu, mbar_wait(&bars->dp_full, i & 1, wd));
       if (!ok) break;
       tc_fence_after();
-      uint32_t da[32], db[32];
-#pragma unroll
-      for (int half = 0; half < 2; half++) {
+      uint32_t dk[32];
+      {
         uint32_t d0[32], d1[32];
-        tmem_ld32(tl + rB + half * 64, d0);
-        tmem_ld32(tl + rB + half * 64 + 32, d1);
+        tmem_ld32(tl + rB + qh, d0);
+        tmem_ld32(tl + rB + qh + 32, d1);
         tmem_ld_wait(d0);
         tmem_ld_wait(d1);
-        if (half == 1) {  // all of dP^T is in registers: region B may take S^T of the next step
-          tc_fence_before();
-          mbar_arrive(&bars->dp_read);
-        }
-        const uint32_t* src = half ? pb : pa;
-        uint32_t* dst = half ? db : da;
+        tc_fence_before();
+        mbar_arrive(&bars->dp_read);  // region B may take S^T of the next step
 #pragma unroll
         for (int c = 0; c < 2; c++) {
           const uint32_t* dv = c ? d1 : d0;
 #pragma unroll
           for (int e4 = 0; e4 < 8; e4++) {
-            const float4 dd = del4[half * 16 + c * 8 + e4];
+            const float4 dd = del4[c * 8 + e4];
             const int w = c * 16 + 2 * e4;
             // bf16 pair -> two floats (first element in the low half)
-            const float p0 = __uint_as_float(src[w] << 16), p1 = __uint_as_float(src[w] & 0xffff0000u);
-            const float p2 = __uint_as_float(src[w + 1] << 16), p3 = __uint_as_float(src[w + 1] & 0xffff0000u);
-            dst[w] = pack_bf16x2(p0 * (__uint_as_float(dv[4 * e4 + 0]) - dd.x),
-                                 p1 * (__uint_as_float(dv[4 * e4 + 1]) - dd.y));
-            dst[w + 1] = pack_bf16x2(p2 * (__uint_as_float(dv[4 * e4 + 2]) - dd.z),
-                                     p3 * (__uint_as_float(dv[4 * e4 + 3]) - dd.w));
+            const float p0 = __uint_as_float(pk[w] << 16), p1 = __uint_as_float(pk[w] & 0xffff0000u);
+            const float p2 = __uint_as_float(pk[w + 1] << 16), p3 = __uint_as_float(pk[w + 1] & 0xffff0000u);
+            dk[w] = pack_bf16x2(p0 * (__uint_as_float(dv[4 * e4 + 0]) - dd.x),
+                                p1 * (__uint_as_float(dv[4 * e4 + 1]) - dd.y));
+            dk[w + 1] = pack_bf16x2(p2 * (__uint_as_float(dv[4 * e4 + 2]) - dd.z),
+                                    p3 * (__uint_as_float(dv[4 * e4 + 3]) - dd.w));
           }
         }
       }
-      // dS^T -> this stage's dO buffer, once dP and dV have finished reading dO.
+      // dS^T -> block wg of this stage's dO buffer, once dP and dV have finished reading dO.
       ok = __all_sync(0xffffffffu, mbar_wait(&bars->dv_done, i & 1, wd));
       if (!ok) break;
-      const uint32_t dsb = smem_u32(sDO) + s * C::TILE;
+      const uint32_t dsb = smem_u32(sDO) + s * C::TILE + wg * C::BLK;
 #pragma unroll
-      for (int c = 0; c < 8; c++) {
-        st_shared_v4(dsb + sw128_offset(r, c), da[4 * c], da[4 * c + 1], da[4 * c + 2], da[4 * c + 3]);
-        st_shared_v4(dsb + C::BLK + sw128_offset(r, c), db[4 * c], db[4 * c + 1], db[4 * c + 2], db[4 * c + 3]);
-      }
+      for (int c = 0; c < 8; c++)
+        st_shared_v4(dsb + sw128_offset(r, c), dk[4 * c], dk[4 * c + 1], dk[4 * c + 2], dk[4 * c + 3]);
       fence_proxy_async_smem();
       mbar_arrive(&bars->dss_full);
     }
@@ -342,11 +368,11 @@ __global__ void __launch_bounds__(320, 1)
     if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&bars->mma_done, 0, wd));
     if (ok) {
       tc_fence_after();
-      __nv_bfloat16* dst = p.dv + ((seq0 + kvc) * p.H + h) * D;
+      __nv_bfloat16* dst = p.dv + ((seq0 + kvc) * p.H + h) * D + qh;
 #pragma unroll 1
-      for (int c = 0; c < D / 32; c++) {
+      for (int c = 0; c < 2; c++) {
         uint32_t v[32];
-        tmem_ld32(tl + C::TM_DV + c * 32, v);
+        tmem_ld32(tl + C::TM_DV + qh + c * 32, v);
         tmem_ld_wait(v);
         if (kv < p.L) {
           uint4* d4 = reinterpret_cast<uint4*>(dst + c * 32);
@@ -360,9 +386,9 @@ __global__ void __launch_bounds__(320, 1)
       }
     }
   } else {
-    // ---------------- dQ drain warps 4-7: thread t <-> TMEM lane t <-> column d = t of dQ^T
-    const int t = threadIdx.x - 128;
-    const uint32_t tl = tmem + ((uint32_t)((warp - 4) * 32) << 16);
+    // ---------------- dQ drain warps 8-11: thread t <-> TMEM lane t <-> column d = t of dQ^T
+    const int t = threadIdx.x - 256;
+    const uint32_t tl = tmem + ((uint32_t)((warp & 3) * 32) << 16);
     bool ok = true;
     for (int i = 0; i < nq; i++) {
       ok = __all_sync(0xffffffffu, mbar_wait(&bars->dq_full, i & 1, wd));
@@ -418,9 +444,11 @@ __global__ void __launch_bounds__(320, 1)
     }
   }
 
+  }
+
   tc_fence_before();
   __syncthreads();
-  if (warp == 8) {
+  if (warp == 12) {
     tc_fence_after();
     tmem_dealloc(tmem, 512);
   }

@@ -267,6 +267,14 @@ __device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr, uint32_t lbo, ui
          ((uint64_t)((sbo >> 4) & 0x3FFFu) << 32) | (1ull << 46) | (2ull << 61);
 }
 
+// A copy of x that the compiler cannot see through (blocks loop-invariant
+// hoisting of values derived from it).
+__device__ __forceinline__ uint64_t opaque_u64(uint64_t x) {
+  uint64_t y;
+  asm volatile("mov.b64 %0, %1;" : "=l"(y) : "l"(x));
+  return y;
+}
+
 // Instruction descriptor for tcgen05.mma.kind::f16: bf16 A/B, fp32 D, dense.
 //   bits 4-5 D type (1 = f32)   7-9 A type (1 = bf16)   10-12 B type (1 = bf16)
 //   bit 15 A MN-major           16 B MN-major           17-22 N >> 3     24-28 M >> 4
@@ -300,6 +308,11 @@ __device__ __forceinline__ float f32x2_hi(uint64_t v) { return __uint_as_float((
 __device__ __forceinline__ uint64_t fma_f32x2(uint64_t a, uint64_t b, uint64_t c) {
   uint64_t d;
   asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ uint64_t mul_f32x2(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
   return d;
 }
 __device__ __forceinline__ uint64_t add_f32x2(uint64_t a, uint64_t b) {
