@@ -71,7 +71,7 @@ typedef struct {
 } dd_attn_desc;
 
 /* Workspace bytes for dd_attn_fwd (for_bwd = 0) or dd_attn_bwd (for_bwd = 1):
- * the status word, and for bwd the fp32 dQ accumulator [B, H, L128, d] plus
+ * the status word, and for bwd the fp32 dQ accumulator (B*H*L128*d floats) plus
  * the per-row D_i and LSE_i*log2(e) vectors [B, H, L128], L128 = L rounded up
  * to a multiple of 128. Returns 0 for an invalid descriptor. */
 size_t dd_attn_workspace_size(const dd_attn_desc* desc, int for_bwd);

@@ -140,8 +140,11 @@ __global__ void __launch_bounds__(256) attn_bwd_post_kernel(const BwdParams p) {
     const long long bi = row / p.H;
     const int i = (int)(bi % p.L);
     const int b = (int)(bi / p.L);
-    const float4* src =
-        reinterpret_cast<const float4*>(p.dq_acc + (((long long)b * p.H + h) * p.L128 + i) * D + part * 8);
+    // d = 64: accumulator rows [B, H, L128, 64]; d = 128: [B, H, 4 chunks, L128, 32]
+    const long long bh = (long long)b * p.H + h;
+    const float* srcf = (D == 128) ? p.dq_acc + ((bh * 4 + (part >> 2)) * p.L128 + i) * 32 + (part & 3) * 8
+                                   : p.dq_acc + (bh * p.L128 + i) * D + part * 8;
+    const float4* src = reinterpret_cast<const float4*>(srcf);
     const float4 x = src[0], y = src[1];
     uint4 w;
     w.x = pack_bf16x2(x.x * p.scale, x.y * p.scale);
@@ -408,41 +411,46 @@ __global__ void __launch_bounds__(320, 1)
     // ---------------- dQ drain warps 4-7 (TMEM lane quarter = warp - 4), then dK rows
     const int t = threadIdx.x - 128;
     const uint32_t tl = tmem + ((uint32_t)((warp - 4) * 32) << 16);
+    // Every drain warp runs the same sequence of named barriers even after an
+    // abort (work is skipped, barriers are not).
     bool ok = true;
     for (int i = 0; i < nq; i++) {
-      ok = __all_sync(0xffffffffu, mbar_wait(&bars->dq_full, i & 1, wd));
-      if (!ok) break;
-      tc_fence_after();
+      ok = __all_sync(0xffffffffu, ok && mbar_wait(&bars->dq_full, i & 1, wd));
       uint32_t v0[32], v1[32];
-      tmem_ld32(tl + C::TM_DQ, v0);
-      tmem_ld32(tl + C::TM_DQ + 32, v1);
-      tmem_ld_wait(v0);
-      tmem_ld_wait(v1);
-      tc_fence_before();
-      mbar_arrive(&bars->dq_free);
+      if (ok) {
+        tc_fence_after();
+        tmem_ld32(tl + C::TM_DQ, v0);
+        tmem_ld32(tl + C::TM_DQ + 32, v1);
+        tmem_ld_wait(v0);
+        tmem_ld_wait(v1);
+        tc_fence_before();
+        mbar_arrive(&bars->dq_free);
+      }
       if (t == 0) bulk_wait_read<0>();  // previous reduction has read the staging tile
       named_bar_sync(1, 128);
-      if constexpr (C::DQ_T) {
-        // thread t holds column d = t for query rows 0..63: staging is [BQ][D] row-major
+      if (ok) {
+        if constexpr (C::DQ_T) {
+          // thread t holds column d = t for query rows 0..63: staging is [BQ][D] row-major
 #pragma unroll
-        for (int e = 0; e < 32; e++) {
-          sDQ[e * D + t] = __uint_as_float(v0[e]);
-          sDQ[(32 + e) * D + t] = __uint_as_float(v1[e]);
-        }
-      } else {
-        // thread t holds query row t, columns d = 0..63
-        float4* row4 = reinterpret_cast<float4*>(sDQ + t * D);
+          for (int e = 0; e < 32; e++) {
+            sDQ[e * D + t] = __uint_as_float(v0[e]);
+            sDQ[(32 + e) * D + t] = __uint_as_float(v1[e]);
+          }
+        } else {
+          // thread t holds query row t, columns d = 0..63
+          float4* row4 = reinterpret_cast<float4*>(sDQ + t * D);
 #pragma unroll
-        for (int e = 0; e < 8; e++) {
-          row4[e] = make_float4(__uint_as_float(v0[4 * e]), __uint_as_float(v0[4 * e + 1]),
-                                __uint_as_float(v0[4 * e + 2]), __uint_as_float(v0[4 * e + 3]));
-          row4[8 + e] = make_float4(__uint_as_float(v1[4 * e]), __uint_as_float(v1[4 * e + 1]),
-                                    __uint_as_float(v1[4 * e + 2]), __uint_as_float(v1[4 * e + 3]));
+          for (int e = 0; e < 8; e++) {
+            row4[e] = make_float4(__uint_as_float(v0[4 * e]), __uint_as_float(v0[4 * e + 1]),
+                                  __uint_as_float(v0[4 * e + 2]), __uint_as_float(v0[4 * e + 3]));
+            row4[8 + e] = make_float4(__uint_as_float(v1[4 * e]), __uint_as_float(v1[4 * e + 1]),
+                                      __uint_as_float(v1[4 * e + 2]), __uint_as_float(v1[4 * e + 3]));
+          }
         }
+        fence_proxy_async_smem();
       }
-      fence_proxy_async_smem();
       named_bar_sync(1, 128);
-      if (t == 0) {
+      if (t == 0 && ok) {
         const int q0 = (m_lo + i) * BQ;
         bulk_reduce_add_f32(p.dq_acc + (vec0 + q0) * D, sDQ, C::DQS_BYTES);
         bulk_commit();

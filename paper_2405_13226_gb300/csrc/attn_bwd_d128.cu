@@ -23,10 +23,13 @@
 // smem: K, V resident; Q, dO, LSE, D in 2 stages. After dV_i (and dP_i) have
 // read dO_i, its buffer receives dS^T_i (bf16, [128 keys][128 queries],
 // 128B-swizzled): the A operand of dK_i (K-major view) and the B operand of
-// dQ^T_i (MN-major view). Warps 4-7 drain dQ^T in four [32 queries x 128] fp32
-// quarters staged in smem, each one cp.reduce.async.bulk .add.f32 into the
-// contiguous accumulator rows (a direct red.global per element was measured
-// slower: its load/store traffic delays the P/dS warps on the same SM).
+// dQ^T_i (MN-major view). The fp32 dQ accumulator is laid out
+// [B, H, 4 column chunks, L128, 32] so that each drain warp (which holds 32 of
+// the d columns of dQ^T) owns a contiguous [32 queries x 32] block per quarter
+// step: it stages that 4 KB block in its own smem slice and adds it with one
+// cp.reduce.async.bulk .add.f32, with no barrier shared between warps (a direct
+// red.global per element was measured slower: its load/store traffic delays
+// the P/dS warps on the same SM).
 //
 // Warp roles, one warpgroup each (thread r of a group <-> key row r <-> TMEM
 // lane r): WG0 / WG1 compute P and dS for query columns 0-63 / 64-127 and write
@@ -388,7 +391,10 @@ __global__ void __launch_bounds__(512, 1)
   } else {
     // ---------------- dQ drain warps 8-11: thread t <-> TMEM lane t <-> column d = t of dQ^T
     const int t = threadIdx.x - 256;
-    const uint32_t tl = tmem + ((uint32_t)((warp & 3) * 32) << 16);
+    const int w = warp & 3;                       // column chunk d = 32 w .. 32 w + 31
+    const uint32_t tl = tmem + ((uint32_t)(w * 32) << 16);
+    float* stg = sSTG + w * (32 * 32);            // this warp's [32 q][32] staging slice
+    float* acc_w = p.dq_acc + (vec0 * 4 + (long long)w * p.L128) * 32;  // chunk w of this (b, h)
     bool ok = true;
     for (int i = 0; i < nq; i++) {
       ok = __all_sync(0xffffffffu, mbar_wait(&bars->dq_full, i & 1, wd));
@@ -405,19 +411,19 @@ __global__ void __launch_bounds__(512, 1)
       const int q0 = (m_lo + i) * BQ;
 #pragma unroll
       for (int c = 0; c < 4; c++) {
-        if (t == 0) bulk_wait_read<0>();  // the previous quarter's reduction has read the staging tile
-        named_bar_sync(1, 128);
+        if (lane == 0) bulk_wait_read<0>();  // this warp's previous reduction has read its slice
+        __syncwarp();
 #pragma unroll
-        for (int e = 0; e < 32; e++) sSTG[e * D + t] = __uint_as_float(v[c][e]);  // row q = 32c + e, col d = t
+        for (int e = 0; e < 32; e++) stg[e * 32 + lane] = __uint_as_float(v[c][e]);  // row q = 32c + e
         fence_proxy_async_smem();
-        named_bar_sync(1, 128);
-        if (t == 0) {
-          bulk_reduce_add_f32(p.dq_acc + (vec0 + q0 + 32 * c) * D, sSTG, C::STG_BYTES);
+        __syncwarp();
+        if (lane == 0) {
+          bulk_reduce_add_f32(acc_w + (long long)(q0 + 32 * c) * 32, stg, 32 * 32 * 4);
           bulk_commit();
         }
       }
     }
-    if (t == 0) bulk_wait<0>();
+    if (lane == 0) bulk_wait<0>();
     // Epilogue: dK rows (scaled).
     if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&bars->mma_done, 0, wd));
     if (ok) {
