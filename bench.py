@@ -36,6 +36,32 @@ T = wl.TOKENS_PER_STEP
 PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
 
+def kernel_source_sha1() -> str:
+    import hashlib
+    h = hashlib.sha1()
+    for f in ("attn_bwd_d128.cu", "common.cuh", "ptx.cuh"):
+        with open(os.path.join(ROOT, "paper_2405_13226_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()
+
+
+def measured_traffic():
+    """Mean DRAM bytes per launch of the backward main kernel over the sweep,
+    from the committed ncu summary, if it was taken on the current sources."""
+    p = os.path.join(ROOT, "profiles", "attn_main_kernels_sweep_traffic.md")
+    if not os.path.exists(p):
+        return None
+    txt = open(p).read()
+    if "source_sha1 (attn_bwd_d128.cu + common.cuh + ptx.cuh): " + kernel_source_sha1() not in txt:
+        return None
+    vals = []
+    for line in txt.splitlines():
+        f = [x.strip() for x in line.split("|")]
+        if len(f) > 5 and f[2] == "attn_bwd_main_d128_kernel":
+            vals.append(float(f[5]))
+    return sum(vals) / len(vals) if vals else None
+
+
 def load_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -280,7 +306,9 @@ def run_ours(args):
     main_ach = main_flops / (main_t * 1e-3) / 1e12
     peak = peaks["bf16_tflops_sustained"]
     roofline = {"kernel": "attn_bwd_main_kernel<128>", "bound": "tensor", "achieved": main_ach, "peak": peak,
-                "unit": "TFLOP/s", "frac": main_ach / peak, "traffic": None,
+                "unit": "TFLOP/s", "frac": main_ach / peak, "traffic": measured_traffic(),
+                "traffic_note": "mean dram__bytes_read+write per launch over the six buckets (ncu, "
+                                "profiles/attn_main_kernels_sweep_traffic.md); null if the kernel changed since",
                 "peak_kind": "bf16_tflops_sustained (%s)" % peak_src,
                 "share_of_step": main_t / total_ms,
                 "fwd_kernel_tflops": sum(bk.flops_fwd for bk in buckets) * args.steps / (fwd_t * 1e-3) / 1e12,
