@@ -5,7 +5,8 @@ call, L in {256, ..., 8192} with B = 65536 / L. One step = forward + backward
 of one 65536-token batch of every bucket (6 calls of each). `value` is the
 algorithmic TFLOP/s over the step (14 d H sum_seq L(L+1)/2 flops per call).
 Also reported: per-bucket ms and TFLOP/s, the document-masked 8x8192
-concat-and-chunk step (16 seeds), the 200-step curriculum stream, the
+concat-and-chunk step (16 seeds), the Pack-8k+DM step, an Algorithm 1
+stream (Grow-P2, 8 cycles), the
 long-context bucket (B=4, L=16384, H=32), the roofline of the dominant kernel,
 an end-to-end number through host buffers, and the fp64 oracle's throughput on
 this host's cores.
@@ -377,9 +378,12 @@ def extra_workloads(ddattn, q, k, v, g, buckets, ws, stream, peaks, dev):
     dm_mean = float(np.mean([x["ms"] for x in dm]))
     out["dm_baseline"] = {"workload": "8 chunks x 8192, H=16, d=128, document-masked, seeds 0..15",
                           "ms_per_step_mean": dm_mean, "per_seed": dm}
-    # curriculum stream: 200 steps, L drawn proportional to DD bucket token counts
+    # Algorithm 1 stream: Grow-P2 odds (Table 2), 8 cycles, bucket token counts
+    # scaled to about 200 full steps of 65536 tokens (whole steps in every cycle)
     counts = wl.dd_bucket_tokens(0)
-    stream_L = wl.curriculum_stream(0, 200, counts)
+    tot = sum(counts.values())
+    sched = {L: max(1, round(c / tot * 25)) * 8 * T for L, c in counts.items()}
+    stream_L = wl.length_curriculum(sched, dict(zip(wl.BUCKETS, wl.CURRICULA["Grow-P2"])), 8, T, seed=0)
     by_L = {bk.L: bk for bk in buckets}
     torch.cuda.synchronize()
     s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -391,12 +395,24 @@ def extra_workloads(ddattn, q, k, v, g, buckets, ws, stream, peaks, dev):
     torch.cuda.synchronize()
     cur_ms = s.elapsed_time(e) / len(stream_L)
     cur_flops = sum(by_L[L].flops for L in stream_L) / len(stream_L)
-    out["curriculum"] = {"workload": "200 steps x 65536 tokens, H=16, d=128; L ~ bucket token share",
-                         "bucket_share": {str(L): c / sum(counts.values()) for L, c in counts.items()},
+    out["curriculum"] = {"workload": "Algorithm 1, Grow-P2 odds, 8 cycles: %d steps x 65536 tokens, H=16, d=128"
+                                     % len(stream_L),
+                         "bucket_steps": {str(L): stream_L.count(L) for L in sorted(sched)},
                          "ms_per_step_mean": cur_ms, "tflops": cur_flops / (cur_ms * 1e-3) / 1e12}
     out["dd_vs_dm_step_time_ratio"] = cur_ms / dm_mean
     out["dd_vs_dm_flop_ratio"] = cur_flops / float(np.mean([
         wl.attn_flops(8, 8192, H, D, wl.concat_and_chunk_offsets(sd)) for sd in range(16)]))
+    # Pack-8k+DM: best-fit-decreasing packing into 8192-token sequences, pad tails masked
+    pk = []
+    for seed in range(4):
+        off_np = wl.packed_dm_offsets(seed)
+        off = torch.from_numpy(off_np).to(dev)
+        bk = Bucket(ddattn, q, k, v, g, 8, 8192, H, offsets=off, ws=ws)
+        ms = time_calls(lambda: (bk.fwd(stream), bk.bwd(stream)), 3, 1, stream)
+        pk.append({"seed": seed, "ms": ms, "pair_fraction": wl.live_pairs(8, 8192, off_np) / wl.live_pairs(8, 8192),
+                   "segments": int(len(wl.segment_lengths(8, 8192, off_np)))})
+    out["pack8k_dm"] = {"workload": "8 best-fit-decreasing bins x 8192, H=16, d=128, document-masked, seeds 0..3",
+                        "ms_per_step_mean": float(np.mean([x["ms"] for x in pk])), "per_seed": pk}
     # long-context bucket: B=4, L=16384, H=32, q/k x3
     qb, kb, vb, gb = wl.attn_inputs(4, 16384, 32, D, seed=0, qk_mult=3.0)
     lq, lk, lv, lg = (to_dev(x, dev) for x in (qb, kb, vb, gb))

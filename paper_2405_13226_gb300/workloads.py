@@ -125,6 +125,98 @@ def curriculum_stream(seed: int = 0, steps: int = 200, bucket_tokens: dict[int, 
     return [int(Ls[i]) for i in idx]
 
 
+# ----------------------------------------------------------------- Algorithm 1
+# Sampling odds over D8..D13 of the paper's curricula (Table 2).
+CURRICULA = {
+    "Uniform": (1, 1, 1, 1, 1, 1),
+    "Grow-Linear": (6, 5, 4, 3, 2, 1),
+    "Grow-P2": (32, 16, 8, 4, 2, 1),
+    "Grow-P100": (100 ** 5, 100 ** 4, 100 ** 3, 100 ** 2, 100, 1),
+    "Shrink-P100": (1, 100, 100 ** 2, 100 ** 3, 100 ** 4, 100 ** 5),
+}
+
+
+def length_curriculum(bucket_tokens: dict[int, int], odds: dict[int, float], cycles: int,
+                      tokens_per_step: int, seed: int = 0) -> list[int]:
+    """Algorithm 1 (length-based sampling and curriculum): sequence length of
+    every optimisation step.
+
+    The n_i tokens of bucket D_i (sequences of length L = 2^i) are split into
+    `cycles` disjoint subsets of n_i / c tokens. In each cycle, while some subset
+    is non-empty: the odds of the non-empty subsets are normalised into
+    probabilities, a bucket i is drawn with them, and b / 2^i sequences are
+    taken from its subset without replacement (fewer if fewer remain)."""
+    rng = _rng(seed, 400)
+    Ls = sorted(bucket_tokens)
+    per_cycle = {}
+    for L in Ls:
+        n_seq = bucket_tokens[L] // L
+        base, extra = divmod(n_seq, cycles)
+        per_cycle[L] = [base + (1 if j < extra else 0) for j in range(cycles)]
+    steps = []
+    for j in range(cycles):
+        left = {L: per_cycle[L][j] for L in Ls}
+        while any(left[L] > 0 for L in Ls):
+            w = np.array([odds[L] if left[L] > 0 else 0.0 for L in Ls], dtype=np.float64)
+            i = int(rng.choice(len(Ls), p=w / w.sum()))
+            L = Ls[i]
+            take = min(left[L], max(tokens_per_step // L, 1))
+            left[L] -= take
+            steps.append(L)
+    return steps
+
+
+# ----------------------------------------------------------------- best-fit packing
+def best_fit_decreasing(chunk_lengths, capacity: int) -> list[list[int]]:
+    """Appendix "Comparison to best-fit sequence packing": chunks (each at most
+    `capacity` tokens) sorted from largest to smallest; each goes to the
+    feasible bin that is left with the least remaining capacity, or to a new
+    bin when none can hold it. Returns the chunk lengths of every bin."""
+    import bisect
+    order = sorted((int(c) for c in chunk_lengths), reverse=True)
+    rem_keys: list[tuple[int, int]] = []      # (remaining capacity, bin id), sorted
+    bins: list[list[int]] = []
+    for c in order:
+        if c > capacity:
+            raise ValueError("chunk longer than the bin capacity")
+        k = bisect.bisect_left(rem_keys, (c, -1))  # smallest remaining >= c
+        if k == len(rem_keys):
+            bins.append([c])
+            bisect.insort(rem_keys, (capacity - c, len(bins) - 1))
+        else:
+            rem, bid = rem_keys.pop(k)
+            bins[bid].append(c)
+            bisect.insort(rem_keys, (rem - c, bid))
+    return bins
+
+
+def packed_dm_offsets(seed: int, n_chunks: int = 8, chunk: int = 8192, n_docs: int = 4000) -> np.ndarray:
+    """Pack-8k+DM workload: lognormal documents cut into pieces of at most
+    `chunk` tokens, packed by best-fit decreasing into `chunk`-token sequences
+    whose unused tail is <PAD>. The first `n_chunks` bins form the step; each
+    document piece and each pad tail is its own masked segment. Returns int32
+    cu_doc_offsets over the n_chunks*chunk tokens."""
+    lengths = lognormal_doc_lengths(_rng(seed, 500), n_docs)
+    pieces = []
+    for ln in lengths:
+        while ln > chunk:
+            pieces.append(chunk)
+            ln -= chunk
+        pieces.append(int(ln))
+    bins = best_fit_decreasing(pieces, chunk)
+    rng = _rng(seed, 501)
+    pick = rng.permutation(len(bins))[:n_chunks]
+    offs = [0]
+    for k, bi in enumerate(pick):
+        pos = k * chunk
+        for c in bins[bi]:
+            pos += c
+            offs.append(pos)
+        if pos < (k + 1) * chunk:          # pad tail
+            offs.append((k + 1) * chunk)
+    return np.unique(np.array(offs, dtype=np.int64)).astype(np.int32)
+
+
 # ----------------------------------------------------------------- statistics
 def segment_lengths(B: int, L: int, cu_doc_offsets=None) -> np.ndarray:
     """Lengths of the attention segments of a step: documents cut at sequence

@@ -107,6 +107,19 @@ def test_dm_baseline_full_size(seed):
         np.testing.assert_array_equal(o_bits[b, i], vb[b, i])
 
 
+@pytest.mark.parametrize("seed", [0, 3])
+def test_pack8k_dm_full_size(seed):
+    """Pack-8k+DM: best-fit-decreasing bins of 8192 tokens with masked pad tails."""
+    off = wl.packed_dm_offsets(seed)
+    qb, kb, vb, gb = _inputs(8, 8192, 16, 128, seed=seed + 20)
+    gpu = run_cuda(qb, kb, vb, gb, default_scale(128), off)
+    errs = check_sampled(qb, kb, vb, gb, default_scale(128), [(0, 0), (5, 9)], off, n_rand=6, gpu=gpu)
+    print(errs)
+    o_bits = gpu[0].view(__import__("torch").int16).cpu().numpy().view(np.uint16)
+    for (b, i) in doc_start_rows(8, 8192, off):
+        np.testing.assert_array_equal(o_bits[b, i], vb[b, i])
+
+
 def test_long_context_full_size():
     """B=4 x L=16384, H=32, d=128, q/k scaled x3 before bf16 rounding."""
     qb, kb, vb, gb = _inputs(4, 16384, 32, 128, qk_mult=3.0)

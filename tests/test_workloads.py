@@ -85,3 +85,77 @@ def test_flop_convention():
     # DD step flops are linear in L at fixed tokens per step
     f = [wl.attn_flops(wl.TOKENS_PER_STEP // L, L, 16, 128) for L in wl.BUCKETS]
     assert f[-1] / f[0] == pytest.approx(8193 / 257)
+
+
+def _run_curriculum(name, cycles, seed=0):
+    counts = {L: 64 * L * 4 for L in wl.BUCKETS}          # 256 sequences' worth of tokens per bucket
+    odds = dict(zip(wl.BUCKETS, wl.CURRICULA[name]))
+    return counts, wl.length_curriculum(counts, odds, cycles, tokens_per_step=8192, seed=seed)
+
+
+@pytest.mark.parametrize("name", list(wl.CURRICULA))
+@pytest.mark.parametrize("cycles", [1, 8])
+def test_algorithm1_consumes_every_bucket_exactly(name, cycles):
+    """Algorithm 1: every token of every bucket is used once; each step is one
+    bucket with b tokens (b / 2^i sequences)."""
+    counts, steps = _run_curriculum(name, cycles)
+    used = {L: 0 for L in wl.BUCKETS}
+    for L in steps:
+        used[L] += 8192
+    assert used == counts
+    assert len(steps) == sum(c // 8192 for c in counts.values())
+
+
+def test_algorithm1_cycles_partition_the_stream():
+    """With c cycles each bucket's subset of a cycle is exhausted before the
+    next cycle starts: the stream splits into c blocks with n_i / c tokens each."""
+    counts, steps = _run_curriculum("Grow-P2", 8)
+    per_cycle_steps = sum(c // 8192 for c in counts.values()) // 8
+    for j in range(8):
+        block = steps[j * per_cycle_steps:(j + 1) * per_cycle_steps]
+        for L in wl.BUCKETS:
+            assert block.count(L) * 8192 == counts[L] // 8
+
+
+def test_algorithm1_curriculum_order():
+    """Grow-P100 draws short sequences first, Shrink-P100 long ones first; the
+    first draw follows the normalised odds."""
+    _, grow = _run_curriculum("Grow-P100", 1)
+    _, shrink = _run_curriculum("Shrink-P100", 1)
+    n = len(grow)
+    assert np.mean(grow[: n // 4]) < np.mean(grow[-n // 4:])
+    assert np.mean(shrink[: n // 4]) > np.mean(shrink[-n // 4:])
+    firsts = [_run_curriculum("Grow-Linear", 1, seed=s)[1][0] for s in range(300)]
+    frac256 = firsts.count(256) / 300            # odds 6 / 21
+    assert abs(frac256 - 6 / 21) < 0.08
+
+
+def test_best_fit_decreasing_against_brute_force():
+    """Best-fit decreasing on small instances: every chunk placed once, no bin
+    over capacity, and each chunk went to the fullest bin that could hold it at
+    that moment (checked by replaying the placement)."""
+    rng = np.random.default_rng(0)
+    for _ in range(50):
+        chunks = rng.integers(1, 20, size=rng.integers(1, 30)).tolist()
+        bins = wl.best_fit_decreasing(chunks, 20)
+        assert sorted(c for b in bins for c in b) == sorted(chunks)
+        assert all(sum(b) <= 20 for b in bins)
+        # replay: bins as lists of remaining capacity in creation order
+        rem = []
+        for c in sorted(chunks, reverse=True):
+            feas = [k for k, r in enumerate(rem) if r >= c]
+            if feas:
+                k = min(feas, key=lambda k: (rem[k] - c, k))
+                rem[k] -= c
+            else:
+                rem.append(20 - c)
+        assert sorted(20 - r for r in rem) == sorted(sum(b) for b in bins)
+
+
+def test_packed_dm_offsets_valid():
+    for seed in range(4):
+        off = wl.packed_dm_offsets(seed)
+        assert off[0] == 0 and off[-1] == 8 * 8192 and np.all(np.diff(off) > 0)
+        assert set(range(0, 8 * 8192 + 1, 8192)) <= set(off.tolist())
+        # packing keeps documents whole far more often than concat-and-chunk
+        assert len(wl.segment_lengths(8, 8192, off)) > 8
