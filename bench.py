@@ -6,7 +6,7 @@ of one 65536-token batch of every bucket (6 calls of each). `value` is the
 algorithmic TFLOP/s over the step (14 d H sum_seq L(L+1)/2 flops per call).
 Also reported: per-bucket ms and TFLOP/s, the document-masked 8x8192
 concat-and-chunk step (16 seeds), the Pack-8k+DM step, an Algorithm 1
-stream (Grow-P2, 8 cycles), the
+stream (Grow-P2, 8 cycles), the sweep with RoPE (f_b = 100k), the
 long-context bucket (B=4, L=16384, H=32), the roofline of the dominant kernel,
 an end-to-end number through host buffers, and the fp64 oracle's throughput on
 this host's cores.
@@ -204,28 +204,38 @@ def to_dev(bits, dev):
 class Bucket:
     """Buffers of one call shape; inputs are views of shared [T, H, D] tensors."""
 
-    def __init__(self, ddattn, q, k, v, g, B, L, Hh, offsets=None, ws=None):
+    def __init__(self, ddattn, q, k, v, g, B, L, Hh, offsets=None, ws=None, rope_base=0.0, qk_rot=None):
         import torch
         self.dd = ddattn
         self.B, self.L = B, L
+        self.rope_base = rope_base
         shape = (B, L, Hh, D)
         self.q, self.k, self.v, self.g = (x.view(shape) for x in (q, k, v, g))
+        if rope_base:
+            # the attention reads the rotated q, k (written by rope_qk each step)
+            self.q_raw, self.k_raw = self.q, self.k
+            self.q, self.k = (x.view(shape) for x in qk_rot)
         self.o = torch.empty_like(self.q)
         self.lse = torch.empty((B, Hh, L), dtype=torch.float32, device=q.device)
         self.dq, self.dk, self.dv = (torch.empty_like(self.q) for _ in range(3))
         self.off = offsets
-        self.desc = ddattn.make_desc(B, L, Hh, D, None, offsets)
+        self.desc = ddattn.make_desc(B, L, Hh, D, None, offsets, rope_base)
         self.ws = ws if ws is not None else ddattn.new_workspace(self.desc, q.device)
         self.flops = wl.attn_flops(B, L, Hh, D, None if offsets is None else offsets.cpu().numpy())
         self.flops_fwd = wl.attn_flops(B, L, Hh, D, None if offsets is None else offsets.cpu().numpy(), bwd=False)
         self.flops_bwd = self.flops - self.flops_fwd
 
+    def rope(self, stream):
+        self.dd.rope_qk(self.q_raw, self.k_raw, self.rope_base, self.q, self.k, stream)
+
     def fwd(self, stream):
+        if self.rope_base:
+            self.rope(stream)
         self.dd.fwd(self.q, self.k, self.v, None, self.off, self.o, self.lse, self.ws, stream)
 
     def bwd(self, stream, phases=None):
         self.dd.bwd(self.q, self.k, self.v, self.o, self.g, self.lse, None, self.off, self.dq, self.dk, self.dv,
-                    self.ws, stream, phases if phases is not None else self.dd.DD_BWD_ALL)
+                    self.ws, stream, phases if phases is not None else self.dd.DD_BWD_ALL, self.rope_base)
 
 
 def run_ours(args):
@@ -413,6 +423,32 @@ def extra_workloads(ddattn, q, k, v, g, buckets, ws, stream, peaks, dev):
                    "segments": int(len(wl.segment_lengths(8, 8192, off_np)))})
     out["pack8k_dm"] = {"workload": "8 best-fit-decreasing bins x 8192, H=16, d=128, document-masked, seeds 0..3",
                         "ms_per_step_mean": float(np.mean([x["ms"] for x in pk])), "per_seed": pk}
+    # RoPE (f_b = 100k) on the bucket sweep: rotation kernel + forward + backward
+    # with R^T fused into the dq / dk outputs, against the same step without RoPE
+    qr, kr = torch.empty_like(q), torch.empty_like(k)
+    rdesc = [ddattn.make_desc(T // L, L, H, D, None, None, 1e5) for L in wl.BUCKETS]
+    rws = ddattn.new_workspace(max(rdesc, key=lambda x: ddattn.workspace_size(x)), dev)
+    rope_rows = []
+    for bk0 in buckets:
+        bk = Bucket(ddattn, q, k, v, g, bk0.B, bk0.L, H, ws=rws, rope_base=1e5, qk_rot=(qr, kr))
+        ms = time_calls(lambda: (bk.fwd(stream), bk.bwd(stream)), 3, 1, stream)
+        ms_plain = time_calls(lambda: (bk0.fwd(stream), bk0.bwd(stream)), 3, 1, stream)
+        rope_ms = time_calls(lambda: bk.rope(stream), 10, 2, stream)
+        rope_rows.append({"L": bk.L, "ms": ms, "ms_without_rope": ms_plain, "rope_kernel_ms": rope_ms,
+                          "rope_kernel_GBps": 4 * T * H * D * 2 / (rope_ms * 1e-3) / 1e9,
+                          "tflops": bk.flops / (ms * 1e-3) / 1e12})
+    st = ddattn.poll_status(rws)
+    if st != 0:
+        raise RuntimeError("device status %d (%s)" % (st, ddattn.status_string(st)))
+    step_rope = sum(x["ms"] for x in rope_rows)
+    step_plain = sum(x["ms_without_rope"] for x in rope_rows)
+    out["rope_sweep"] = {"workload": "bucket sweep with RoPE f_b=100k: dd_rope_qk + fwd + bwd per bucket",
+                         "ms_per_step": step_rope, "ms_per_step_without_rope": step_plain,
+                         "overhead": step_rope / step_plain - 1.0,
+                         "rope_kernel_frac_of_measured_hbm": float(np.median([x["rope_kernel_GBps"] for x in rope_rows]))
+                         / peaks["hbm_gbs"],
+                         "per_bucket": rope_rows}
+    del qr, kr, rws
     # long-context bucket: B=4, L=16384, H=32, q/k x3
     qb, kb, vb, gb = wl.attn_inputs(4, 16384, 32, D, seed=0, qk_mult=3.0)
     lq, lk, lv, lg = (to_dev(x, dev) for x in (qb, kb, vb, gb))

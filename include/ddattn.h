@@ -18,6 +18,19 @@
  *     dq_i = scale sum_j dS_ij k_j, dk_j = scale sum_i dS_ij q_i,
  *     dv_j = sum_i P_ij dO_i.
  *
+ * Rotary position embedding (Sec. 3, training setup; base frequency f_b of
+ * the f_b ablation table and Table 2): before attention, consecutive
+ * components of every q and k head vector are rotated by the token's position
+ * m inside its sequence,
+ *     theta_j = f_b^(-2j/d),
+ *     (x_2j, x_2j+1) -> (x_2j cos m theta_j - x_2j+1 sin m theta_j,
+ *                        x_2j sin m theta_j + x_2j+1 cos m theta_j).
+ *   dd_rope_qk applies it (bf16 out). With desc->rope_base = f_b > 0, the
+ *   q and k given to dd_attn_fwd / dd_attn_bwd are the ROTATED ones, and
+ *   dd_attn_bwd returns dq, dk with respect to the UN-rotated q and k (it
+ *   applies the transposed rotation to the rotated-space gradients inside its
+ *   kernels). rope_base = 0 means no rotation.
+ *
  * Layouts (all device memory, caller-owned, never freed or kept by the library):
  *   q, k, v, o, dO, dq, dk, dv : bf16, [B, L, H, d] contiguous (token-major).
  *   lse                        : fp32, [B, H, L] contiguous, natural log.
@@ -68,20 +81,34 @@ typedef struct {
   float scale;                     /* softmax scale, usually 1/sqrt(d); finite */
   const int32_t* cu_doc_offsets;   /* DEVICE pointer or NULL (plain causal) */
   int32_t n_offsets;               /* entries of cu_doc_offsets (>= 2 when non-NULL) */
+  float rope_base;                 /* RoPE base frequency f_b; 0 = no RoPE; else finite and > 0 */
 } dd_attn_desc;
 
 /* Workspace bytes for dd_attn_fwd (for_bwd = 0) or dd_attn_bwd (for_bwd = 1):
  * the status word, and for bwd the fp32 dQ accumulator (B*H*L128*d floats) plus
  * the per-row D_i and LSE_i*log2(e) vectors [B, H, L128], L128 = L rounded up
- * to a multiple of 128. Returns 0 for an invalid descriptor. */
+ * to a multiple of 128, plus, when rope_base > 0, a [L, d/2] table of
+ * (cos, sin) pairs (fp32). Returns 0 for an invalid descriptor. */
 size_t dd_attn_workspace_size(const dd_attn_desc* desc, int for_bwd);
 
 /* Forward (Sec. 2.2 step; mask per cu_doc_offsets): writes o and lse. */
 dd_status dd_attn_fwd(const dd_attn_desc* desc, const void* q, const void* k, const void* v, void* o, float* lse,
                       void* ws, size_t ws_bytes, void* stream);
 
+/* Rotary position embedding of q and k (see the top of this file): writes
+ * q_rot = R q and k_rot = R k, bf16, [B, L, H, d] like q and k, computed in
+ * fp32 from the bf16 inputs and rounded to nearest-even. Needs
+ * desc->rope_base > 0; the mask fields of desc are ignored (positions restart
+ * at every sequence, not at every document: RoPE scores depend on m - n only,
+ * so inside a document the two choices agree). In place (q_rot == q,
+ * k_rot == k) is allowed. One bandwidth-bound kernel, no workspace. */
+dd_status dd_rope_qk(const dd_attn_desc* desc, const void* q, const void* k, void* q_rot, void* k_rot,
+                     void* stream);
+
 /* Backward: from q, k, v, the forward's o and lse, and dO, writes dq, dk, dv
- * (bf16, overwritten, not accumulated). Recomputes P from lse. */
+ * (bf16, overwritten, not accumulated). Recomputes P from lse. With
+ * rope_base > 0, q and k are the rotated ones and dq, dk are returned with
+ * respect to the un-rotated q, k. */
 dd_status dd_attn_bwd(const dd_attn_desc* desc, const void* q, const void* k, const void* v, const void* o,
                       const void* dO, const float* lse, void* dq, void* dk, void* dv, void* ws, size_t ws_bytes,
                       void* stream);
@@ -89,7 +116,9 @@ dd_status dd_attn_bwd(const dd_attn_desc* desc, const void* q, const void* k, co
 /* The backward as its three kernels, for callers that time or schedule them
  * separately: DD_BWD_PRE (D_i, padded LSE, zero the dQ accumulator in ws),
  * DD_BWD_MAIN (P recompute and the five contractions; dK, dV and the fp32 dQ
- * accumulator), DD_BWD_POST (dq = bf16(scale * accumulator)). `phases` is a
+ * accumulator), DD_BWD_POST (dq = bf16(scale * accumulator)). With RoPE the
+ * PRE phase also fills the (cos, sin) table, and MAIN / POST rotate dk / dq
+ * back with it. `phases` is a
  * bit mask; issuing the phases in this order, with the same arguments and
  * workspace, equals one dd_attn_bwd call (dd_attn_bwd = all three). */
 enum { DD_BWD_PRE = 1, DD_BWD_MAIN = 2, DD_BWD_POST = 4, DD_BWD_ALL = 7 };

@@ -29,7 +29,22 @@ dd_status check_desc(const dd_attn_desc* d) {
     if (d->n_offsets < 2 || (reinterpret_cast<uintptr_t>(d->cu_doc_offsets) & 3u)) return DD_ERR_INVALID_ARG;
     if ((long long)d->B * d->L > 2147483647LL) return DD_ERR_INVALID_ARG;  // int32 offsets
   }
+  if (!std::isfinite(d->rope_base) || d->rope_base < 0.f) return DD_ERR_INVALID_ARG;
+  if (d->rope_base > 0.f && d->L > (1 << 24)) return DD_ERR_INVALID_ARG;  // positions exact in fp32
   return DD_OK;
+}
+
+bool has_rope(const dd_attn_desc* d) { return d->rope_base > 0.f; }
+
+// theta_j = f_b^(-2j/d) in double, split into fp32 head + fp32 remainder.
+RopeFreq rope_freq(const dd_attn_desc* d) {
+  RopeFreq f{};
+  for (int j = 0; j < d->d / 2; j++) {
+    const double th = std::pow((double)d->rope_base, -2.0 * j / d->d);
+    f.hi[j] = (float)th;
+    f.lo[j] = (float)(th - (double)f.hi[j]);
+  }
+  return f;
 }
 
 size_t bwd_vec_bytes(const dd_attn_desc* d) {
@@ -37,6 +52,9 @@ size_t bwd_vec_bytes(const dd_attn_desc* d) {
 }
 size_t bwd_acc_bytes(const dd_attn_desc* d) {
   return align256((size_t)d->B * d->H * round128(d->L) * d->d * sizeof(float));
+}
+size_t rope_tab_bytes(const dd_attn_desc* d) {
+  return has_rope(d) ? align256((size_t)d->L * (d->d / 2) * sizeof(float2)) : 0;
 }
 
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
@@ -122,7 +140,28 @@ extern "C" {
 size_t dd_attn_workspace_size(const dd_attn_desc* desc, int for_bwd) {
   if (check_desc(desc) != DD_OK) return 0;
   if (!for_bwd) return kStatusBytes;
-  return kStatusBytes + 2 * bwd_vec_bytes(desc) + bwd_acc_bytes(desc);
+  return kStatusBytes + 2 * bwd_vec_bytes(desc) + bwd_acc_bytes(desc) + rope_tab_bytes(desc);
+}
+
+dd_status dd_rope_qk(const dd_attn_desc* desc, const void* q, const void* k, void* q_rot, void* k_rot,
+                     void* stream) {
+  dd_status st = check_desc(desc);
+  if (st != DD_OK) return st;
+  if (!has_rope(desc)) return DD_ERR_INVALID_ARG;
+  if (!q || !k || !q_rot || !k_rot) return DD_ERR_INVALID_ARG;
+  if (!aligned16(q) || !aligned16(k) || !aligned16(q_rot) || !aligned16(k_rot)) return DD_ERR_INVALID_ARG;
+  if ((st = check_device()) != DD_OK) return st;
+  RopeParams p;
+  p.rows = (long long)desc->B * desc->L;
+  p.L = desc->L;
+  p.H = desc->H;
+  p.d = desc->d;
+  p.q = static_cast<const __nv_bfloat16*>(q);
+  p.k = static_cast<const __nv_bfloat16*>(k);
+  p.q_rot = static_cast<__nv_bfloat16*>(q_rot);
+  p.k_rot = static_cast<__nv_bfloat16*>(k_rot);
+  p.f = rope_freq(desc);
+  return launch_rope_qk(p, static_cast<cudaStream_t>(stream)) == cudaSuccess ? DD_OK : DD_ERR_CUDA;
 }
 
 dd_status dd_attn_fwd(const dd_attn_desc* desc, const void* q, const void* k, const void* v, void* o, float* lse,
@@ -198,6 +237,10 @@ dd_status dd_attn_bwd_phases(const dd_attn_desc* desc, const void* q, const void
   p.dq = static_cast<__nv_bfloat16*>(dq);
   p.dk = static_cast<__nv_bfloat16*>(dk);
   p.dv = static_cast<__nv_bfloat16*>(dv);
+  p.rope_tab = has_rope(desc) ? reinterpret_cast<float2*>(w + kStatusBytes + 2 * bwd_vec_bytes(desc) +
+                                                           bwd_acc_bytes(desc))
+                              : nullptr;
+  p.rope = has_rope(desc) ? rope_freq(desc) : RopeFreq{};
   p.status = static_cast<int*>(ws);
   p.timeout_ns = wait_limit_ns();
   cudaError_t e = launch_attn_bwd(desc->d, tq, tk, tv, tdo, p, phases, static_cast<cudaStream_t>(stream));

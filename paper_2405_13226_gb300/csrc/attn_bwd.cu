@@ -16,7 +16,9 @@
 //                  dQ is drained by a second warpgroup through smem into one
 //                  bulk cp.reduce.async.bulk .add.f32 of the contiguous
 //                  [BQ x d] block of the fp32 accumulator.
-//   attn_bwd_post  dq = bf16(scale * dQacc).
+//   attn_bwd_post  dq = bf16(scale * dQacc), rotated back (R^T) with RoPE.
+// With RoPE the pre phase also fills the [L, d/2] (cos, sin) table and the dK
+// epilogue rotates dk back with it.
 // Warp roles of attn_bwd_main: warps 0-3 compute P/dS (thread r <-> key row r
 // <-> TMEM lane r) and write dV; warps 4-7 drain dQ and write dK; warp 8 is
 // the TMA producer; warp 9 issues tcgen05.mma.
@@ -146,11 +148,21 @@ __global__ void __launch_bounds__(256) attn_bwd_post_kernel(const BwdParams p) {
                                    : p.dq_acc + (bh * p.L128 + i) * D + part * 8;
     const float4* src = reinterpret_cast<const float4*>(srcf);
     const float4 x = src[0], y = src[1];
+    float f[8] = {x.x * p.scale, x.y * p.scale, x.z * p.scale, x.w * p.scale,
+                  y.x * p.scale, y.y * p.scale, y.z * p.scale, y.w * p.scale};
+    if (p.rope_tab) {  // dq = R^T dq_rot: pairs j = 4 part .. 4 part + 3 at position i
+      const float4* t4 = reinterpret_cast<const float4*>(p.rope_tab + (long long)i * (D / 2) + part * 4);
+      const float4 a = t4[0], c = t4[1];
+      rope_unrotate_pair(f[0], f[1], a.x, a.y);
+      rope_unrotate_pair(f[2], f[3], a.z, a.w);
+      rope_unrotate_pair(f[4], f[5], c.x, c.y);
+      rope_unrotate_pair(f[6], f[7], c.z, c.w);
+    }
     uint4 w;
-    w.x = pack_bf16x2(x.x * p.scale, x.y * p.scale);
-    w.y = pack_bf16x2(x.z * p.scale, x.w * p.scale);
-    w.z = pack_bf16x2(y.x * p.scale, y.y * p.scale);
-    w.w = pack_bf16x2(y.z * p.scale, y.w * p.scale);
+    w.x = pack_bf16x2(f[0], f[1]);
+    w.y = pack_bf16x2(f[2], f[3]);
+    w.z = pack_bf16x2(f[4], f[5]);
+    w.w = pack_bf16x2(f[6], f[7]);
     reinterpret_cast<uint4*>(p.dq + row * D)[part] = w;
   }
 }
@@ -464,21 +476,12 @@ __global__ void __launch_bounds__(320, 1)
       const int kv = kv0 + t;
       const int kvc = kv < p.L ? kv : p.L - 1;
       __nv_bfloat16* dst = p.dk + ((seq0 + kvc) * p.H + h) * D;
-      const float sc = p.scale;
 #pragma unroll 1
       for (int c = 0; c < D / 32; c++) {
         uint32_t v[32];
         tmem_ld32(tl + C::TM_DK + c * 32, v);
         tmem_ld_wait(v);
-        if (kv < p.L) {
-          uint4* d4 = reinterpret_cast<uint4*>(dst + c * 32);
-#pragma unroll
-          for (int q = 0; q < 4; q++)
-            d4[q] = make_uint4(pack_bf16x2(__uint_as_float(v[8 * q]) * sc, __uint_as_float(v[8 * q + 1]) * sc),
-                               pack_bf16x2(__uint_as_float(v[8 * q + 2]) * sc, __uint_as_float(v[8 * q + 3]) * sc),
-                               pack_bf16x2(__uint_as_float(v[8 * q + 4]) * sc, __uint_as_float(v[8 * q + 5]) * sc),
-                               pack_bf16x2(__uint_as_float(v[8 * q + 6]) * sc, __uint_as_float(v[8 * q + 7]) * sc));
-        }
+        if (kv < p.L) store_dk_row32(dst + c * 32, v, p.scale, p.rope_tab, kv, D / 2, c * 16);
       }
     }
   }
@@ -513,6 +516,7 @@ static cudaError_t launch_bwd_d(const CUtensorMap& tq, const CUtensorMap& tk, co
   const int ew_blocks = (int)std::min<long long>((work + 255) / 256, (long long)nsm * 8);
   cudaError_t e = cudaSuccess;
   if (phases & 1) {
+    if (p.rope_tab && (e = launch_rope_table(p.L, D, p.rope, p.rope_tab, stream)) != cudaSuccess) return e;
     attn_bwd_pre_kernel<D><<<ew_blocks, 256, 0, stream>>>(p);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }

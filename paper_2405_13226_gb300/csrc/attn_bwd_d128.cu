@@ -431,21 +431,12 @@ __global__ void __launch_bounds__(512, 1)
       const int kv = kv0 + t;
       const int kvc = kv < p.L ? kv : p.L - 1;
       __nv_bfloat16* dst = p.dk + ((seq0 + kvc) * p.H + h) * D;
-      const float sc = p.scale;
 #pragma unroll 1
       for (int c = 0; c < D / 32; c++) {
         uint32_t v[32];
         tmem_ld32(tl + C::TM_DK + c * 32, v);
         tmem_ld_wait(v);
-        if (kv < p.L) {
-          uint4* d4 = reinterpret_cast<uint4*>(dst + c * 32);
-#pragma unroll
-          for (int q = 0; q < 4; q++)
-            d4[q] = make_uint4(pack_bf16x2(__uint_as_float(v[8 * q]) * sc, __uint_as_float(v[8 * q + 1]) * sc),
-                               pack_bf16x2(__uint_as_float(v[8 * q + 2]) * sc, __uint_as_float(v[8 * q + 3]) * sc),
-                               pack_bf16x2(__uint_as_float(v[8 * q + 4]) * sc, __uint_as_float(v[8 * q + 5]) * sc),
-                               pack_bf16x2(__uint_as_float(v[8 * q + 6]) * sc, __uint_as_float(v[8 * q + 7]) * sc));
-        }
+        if (kv < p.L) store_dk_row32(dst + c * 32, v, p.scale, p.rope_tab, kv, D / 2, c * 16);
       }
     }
   }

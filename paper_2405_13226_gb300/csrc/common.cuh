@@ -60,6 +60,59 @@ __device__ __forceinline__ void mbar_wait_drain(uint64_t* bar, uint32_t parity, 
   }
 }
 
+// RoPE frequencies theta_j = f_b^(-2j/d), j < d/2 <= 64, each split into an
+// fp32 head and the fp32 rounding of its remainder (computed on the host in
+// double precision).
+struct RopeFreq {
+  float hi[64], lo[64];
+};
+
+// (cos, sin) of m * theta_j for an integer position m < 2^24. The product is
+// taken as p + e, p = fl(m * hi) and e = its exact rounding error (one fma)
+// plus m * lo; sincosf gets the representable p, and the small e (|e| < ulp(p))
+// is added by the angle-sum identity with cos e = 1 - e^2/2, sin e = e.
+__device__ __forceinline__ float2 rope_cos_sin(int m, float hi, float lo) {
+  const float fm = (float)m;
+  const float p = fm * hi;
+  float e = fmaf(fm, hi, -p);
+  e = fmaf(fm, lo, e);
+  float s, c;
+  sincosf(p, &s, &c);
+  const float h = 0.5f * e * e;
+  return make_float2(fmaf(-e, s, fmaf(-h, c, c)), fmaf(e, c, fmaf(-h, s, s)));
+}
+
+// g <- R^T g for one rotated pair (cs = (cos, sin)).
+__device__ __forceinline__ void rope_unrotate_pair(float& g0, float& g1, float c, float s) {
+  const float a = fmaf(g0, c, g1 * s);
+  const float b = fmaf(g1, c, -g0 * s);
+  g0 = a;
+  g1 = b;
+}
+
+// One 32-column slice of a dK row: dk = scale * acc, then R^T at position m
+// when tab != nullptr (pairs j0 .. j0 + 15 of a row of `half` table entries).
+__device__ __forceinline__ void store_dk_row32(__nv_bfloat16* dst, const uint32_t (&v)[32], float sc,
+                                               const float2* tab, int m, int half, int j0) {
+  float f[32];
+#pragma unroll
+  for (int e = 0; e < 32; e++) f[e] = __uint_as_float(v[e]) * sc;
+  if (tab) {
+    const float4* t4 = reinterpret_cast<const float4*>(tab + (long long)m * half + j0);
+#pragma unroll
+    for (int u = 0; u < 8; u++) {
+      const float4 cs = t4[u];
+      rope_unrotate_pair(f[4 * u], f[4 * u + 1], cs.x, cs.y);
+      rope_unrotate_pair(f[4 * u + 2], f[4 * u + 3], cs.z, cs.w);
+    }
+  }
+  uint4* d4 = reinterpret_cast<uint4*>(dst);
+#pragma unroll
+  for (int q = 0; q < 4; q++)
+    d4[q] = make_uint4(pack_bf16x2(f[8 * q], f[8 * q + 1]), pack_bf16x2(f[8 * q + 2], f[8 * q + 3]),
+                       pack_bf16x2(f[8 * q + 4], f[8 * q + 5]), pack_bf16x2(f[8 * q + 6], f[8 * q + 7]));
+}
+
 struct FwdParams {
   int B, L, H, nqt;
   float scale_log2;  // softmax scale * log2(e)
@@ -85,16 +138,30 @@ struct BwdParams {
   __nv_bfloat16* dq;
   __nv_bfloat16* dk;
   __nv_bfloat16* dv;
+  float2* rope_tab;  // [L, d/2] (cos, sin) of m theta_j, or nullptr without RoPE
+  RopeFreq rope;     // frequencies that fill rope_tab
   int* status;
   unsigned long long timeout_ns;
 };
 
-// Launchers (defined in attn_fwd.cu / attn_bwd.cu); return a cudaError_t.
+struct RopeParams {
+  long long rows;  // B * L token rows
+  int L, H, d;
+  const __nv_bfloat16* q;
+  const __nv_bfloat16* k;
+  __nv_bfloat16* q_rot;
+  __nv_bfloat16* k_rot;
+  RopeFreq f;
+};
+
+// Launchers (defined in attn_fwd.cu / attn_bwd.cu / rope.cu); return a cudaError_t.
 cudaError_t launch_attn_fwd(int d, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
                             const FwdParams& p, cudaStream_t stream);
 cudaError_t launch_attn_bwd_main_d128(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
                                       const CUtensorMap& tdo, const BwdParams& p, cudaStream_t stream);
 cudaError_t launch_attn_bwd(int d, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
                             const CUtensorMap& tdo, const BwdParams& p, int phases, cudaStream_t stream);
+cudaError_t launch_rope_qk(const RopeParams& p, cudaStream_t stream);
+cudaError_t launch_rope_table(int L, int d, const RopeFreq& f, float2* tab, cudaStream_t stream);
 
 }  // namespace ddattn

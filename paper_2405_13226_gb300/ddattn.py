@@ -27,13 +27,15 @@ class DDAttnError(RuntimeError):
 
 class Desc(ctypes.Structure):
     _fields_ = [("B", ctypes.c_int32), ("L", ctypes.c_int32), ("H", ctypes.c_int32), ("d", ctypes.c_int32),
-                ("scale", ctypes.c_float), ("cu_doc_offsets", ctypes.c_void_p), ("n_offsets", ctypes.c_int32)]
+                ("scale", ctypes.c_float), ("cu_doc_offsets", ctypes.c_void_p), ("n_offsets", ctypes.c_int32),
+                ("rope_base", ctypes.c_float)]
 
 
 _lib = None
 
 EXPORTS = ("dd_attn_workspace_size", "dd_attn_fwd", "dd_attn_bwd", "dd_attn_bwd_phases", "dd_attn_bwd_noalloc",
-           "dd_attn_clear_status", "dd_attn_poll_status", "dd_selftest_wait_timeout", "dd_status_string")
+           "dd_rope_qk", "dd_attn_clear_status", "dd_attn_poll_status", "dd_selftest_wait_timeout",
+           "dd_status_string")
 NOALLOC_SCRATCH_BYTES = 32 << 20
 DD_BWD_PRE, DD_BWD_MAIN, DD_BWD_POST, DD_BWD_ALL = 1, 2, 4, 7
 
@@ -58,6 +60,8 @@ def lib() -> ctypes.CDLL:
         L.dd_attn_bwd_phases.restype = i32
         L.dd_attn_bwd_noalloc.argtypes = [dp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp]
         L.dd_attn_bwd_noalloc.restype = i32
+        L.dd_rope_qk.argtypes = [dp, vp, vp, vp, vp, vp]
+        L.dd_rope_qk.restype = i32
         L.dd_attn_clear_status.argtypes = [vp, vp]
         L.dd_attn_clear_status.restype = i32
         L.dd_attn_poll_status.argtypes = [vp]
@@ -74,14 +78,15 @@ def status_string(s: int) -> str:
     return lib().dd_status_string(int(s)).decode()
 
 
-def make_desc(B: int, L: int, H: int, d: int, scale: float | None = None, cu_doc_offsets=None) -> Desc:
+def make_desc(B: int, L: int, H: int, d: int, scale: float | None = None, cu_doc_offsets=None,
+              rope_base: float = 0.0) -> Desc:
     if scale is None:
         scale = 1.0 / math.sqrt(d)
     off_ptr, n_off = None, 0
     if cu_doc_offsets is not None:
         assert cu_doc_offsets.dtype == torch.int32 and cu_doc_offsets.is_cuda and cu_doc_offsets.is_contiguous()
         off_ptr, n_off = cu_doc_offsets.data_ptr(), cu_doc_offsets.numel()
-    return Desc(B, L, H, d, float(scale), off_ptr, n_off)
+    return Desc(B, L, H, d, float(scale), off_ptr, n_off, float(rope_base))
 
 
 def workspace_size(desc: Desc, for_bwd: bool = True) -> int:
@@ -109,8 +114,25 @@ def _check_qkv(*ts):
             raise ValueError("expected contiguous CUDA bf16 tensors of shape [B, L, H, d]")
 
 
+def rope_qk(q, k, rope_base, q_rot=None, k_rot=None, stream=None):
+    """q_rot, k_rot = RoPE(q), RoPE(k) with base frequency rope_base (in place
+    if q_rot is q / k_rot is k)."""
+    _check_qkv(q, k)
+    B, L, H, d = q.shape
+    desc = make_desc(B, L, H, d, None, None, rope_base)
+    q_rot = torch.empty_like(q) if q_rot is None else q_rot
+    k_rot = torch.empty_like(k) if k_rot is None else k_rot
+    _check_qkv(q_rot, k_rot)
+    st = lib().dd_rope_qk(ctypes.byref(desc), q.data_ptr(), k.data_ptr(), q_rot.data_ptr(), k_rot.data_ptr(),
+                          _stream(stream))
+    if st != DD_OK:
+        raise DDAttnError(st, "dd_rope_qk")
+    return q_rot, k_rot
+
+
 def fwd(q, k, v, scale=None, cu_doc_offsets=None, out=None, lse=None, workspace=None, stream=None):
-    """o, lse = attention forward (causal; document-masked if cu_doc_offsets)."""
+    """o, lse = attention forward (causal; document-masked if cu_doc_offsets).
+    With RoPE, q and k are the rotated tensors from rope_qk."""
     _check_qkv(q, k, v)
     B, L, H, d = q.shape
     desc = make_desc(B, L, H, d, scale, cu_doc_offsets)
@@ -128,12 +150,14 @@ def fwd(q, k, v, scale=None, cu_doc_offsets=None, out=None, lse=None, workspace=
 
 
 def bwd(q, k, v, o, dO, lse, scale=None, cu_doc_offsets=None, dq=None, dk=None, dv=None, workspace=None,
-        stream=None, phases=DD_BWD_ALL):
+        stream=None, phases=DD_BWD_ALL, rope_base=0.0):
     """dq, dk, dv = attention backward from the forward's o and lse (`phases`:
-    a subset of its three kernels, see dd_attn_bwd_phases)."""
+    a subset of its three kernels, see dd_attn_bwd_phases). With rope_base > 0,
+    q and k are the rotated tensors and dq, dk are returned with respect to the
+    un-rotated ones."""
     _check_qkv(q, k, v, o, dO)
     B, L, H, d = q.shape
-    desc = make_desc(B, L, H, d, scale, cu_doc_offsets)
+    desc = make_desc(B, L, H, d, scale, cu_doc_offsets, rope_base)
     dq = torch.empty_like(q) if dq is None else dq
     dk = torch.empty_like(k) if dk is None else dk
     dv = torch.empty_like(v) if dv is None else dv

@@ -7,6 +7,7 @@ import math
 import numpy as np
 
 from oracle import oracle as orc
+from oracle import rope
 from paper_2405_13226_gb300 import workloads as wl
 
 # Tolerances: bf16 inputs, fp32 accumulation (O: max abs and relative L2; grads: relative L2).
@@ -38,37 +39,51 @@ def bits_f64(bits) -> np.ndarray:
     return wl.bf16_bits_to_f32(bits).astype(np.float64)
 
 
-def run_cuda(qb, kb, vb, gb, scale, offsets=None, device="cuda"):
-    """fwd + bwd through the C ABI on bf16 bit arrays [B, L, H, d]."""
+def run_cuda(qb, kb, vb, gb, scale, offsets=None, device="cuda", rope_base=0.0):
+    """fwd + bwd through the C ABI on bf16 bit arrays [B, L, H, d] (with
+    rope_base > 0: rope_qk first, and dq, dk with respect to the un-rotated q, k)."""
     import torch
     from paper_2405_13226_gb300 import ddattn
     q, k, v, g = (to_device(x, device) for x in (qb, kb, vb, gb))
     off = None if offsets is None else torch.from_numpy(np.asarray(offsets, np.int32)).to(device)
     B, L, H, d = q.shape
-    desc = ddattn.make_desc(B, L, H, d, scale, off)
+    desc = ddattn.make_desc(B, L, H, d, scale, off, rope_base)
     ws = ddattn.new_workspace(desc, q.device, for_bwd=True)
+    if rope_base:
+        q, k = ddattn.rope_qk(q, k, rope_base)
     o, lse = ddattn.fwd(q, k, v, scale, off, workspace=ws)
-    dq, dk, dv = ddattn.bwd(q, k, v, o, g, lse, scale, off, workspace=ws)
+    dq, dk, dv = ddattn.bwd(q, k, v, o, g, lse, scale, off, workspace=ws, rope_base=rope_base)
     torch.cuda.synchronize()
     st = ddattn.poll_status(ws)
     assert st == 0, "device status %d" % st
     return o, lse, dq, dk, dv
 
 
-def oracle_full(qb, kb, vb, gb, scale, offsets=None):
+def rope_inputs(q, k, rope_base):
+    """[B, L, H, d] float64 q, k -> the bf16-rounded rotated q, k the attention sees."""
+    return rope.round_to_bf16(rope.rope_rotate(q, rope_base)), rope.round_to_bf16(rope.rope_rotate(k, rope_base))
+
+
+def oracle_full(qb, kb, vb, gb, scale, offsets=None, rope_base=0.0):
     """Oracle over every (b, h) slice. Returns arrays in [B, L, H, d] / [B, H, L]."""
     B, L, H, d = qb.shape
-    q, k, v, g = (bits_f64(x).transpose(0, 2, 1, 3).reshape(B * H, L, d) for x in (qb, kb, vb, gb))
+    q, k, v, g = (bits_f64(x) for x in (qb, kb, vb, gb))
+    if rope_base:
+        q, k = rope_inputs(q, k, rope_base)
+    q, k, v, g = (x.transpose(0, 2, 1, 3).reshape(B * H, L, d) for x in (q, k, v, g))
     doc = np.stack([orc.doc_ids(L, b, offsets) for b in range(B) for _ in range(H)])
     o, lse = orc.attn_fwd(q, k, v, doc, scale)
     dq, dk, dv = orc.attn_bwd(q, k, v, g, doc, scale)
     back = lambda x: x.reshape(B, H, L, d).transpose(0, 2, 1, 3)
-    return back(o), lse.reshape(B, H, L), back(dq), back(dk), back(dv)
+    dq, dk = back(dq), back(dk)
+    if rope_base:
+        dq, dk = rope.rope_unrotate(dq, rope_base), rope.rope_unrotate(dk, rope_base)
+    return back(o), lse.reshape(B, H, L), dq, dk, back(dv)
 
 
-def check_full(qb, kb, vb, gb, scale, offsets=None):
-    o, lse, dq, dk, dv = run_cuda(qb, kb, vb, gb, scale, offsets)
-    ro, rlse, rdq, rdk, rdv = oracle_full(qb, kb, vb, gb, scale, offsets)
+def check_full(qb, kb, vb, gb, scale, offsets=None, rope_base=0.0):
+    o, lse, dq, dk, dv = run_cuda(qb, kb, vb, gb, scale, offsets, rope_base=rope_base)
+    ro, rlse, rdq, rdk, rdv = oracle_full(qb, kb, vb, gb, scale, offsets, rope_base)
     go = to_f64(o)
     errs = {
         "o_max": float(np.abs(go - ro).max()),
@@ -92,20 +107,28 @@ def sample_rows(L: int, n_rand: int, seed: int) -> np.ndarray:
     return np.array(sorted({r for r in fixed + rnd if 0 <= r < L}), dtype=np.int32)
 
 
-def check_sampled(qb, kb, vb, gb, scale, slices, offsets=None, n_rand=8, gpu=None):
+def check_sampled(qb, kb, vb, gb, scale, slices, offsets=None, n_rand=8, gpu=None, rope_base=0.0):
     """Full-size GPU run (or `gpu` results), oracle on sampled rows of (b, h) slices."""
     if gpu is None:
-        gpu = run_cuda(qb, kb, vb, gb, scale, offsets)
+        gpu = run_cuda(qb, kb, vb, gb, scale, offsets, rope_base=rope_base)
     o, lse, dq, dk, dv = (to_f64(t) for t in gpu)
     B, L, H, d = qb.shape
     acc = {k: ([], []) for k in ("o", "lse", "dq", "dk", "dv")}
     for (b, h) in slices:
         sl = lambda x: bits_f64(x[b, :, h, :])
         q, k, v, g = sl(qb), sl(kb), sl(vb), sl(gb)
+        if rope_base:
+            q, k = (x[0, :, 0] for x in rope_inputs(q[None, :, None], k[None, :, None], rope_base))
         doc = orc.doc_ids(L, b, offsets)
         rows = sample_rows(L, n_rand, seed=b * 1000 + h)
         ro, rlse = orc.attn_fwd_rows(q, k, v, doc, scale, rows)
         rdq, rdk, rdv = orc.attn_bwd_rows(q, k, v, g, doc, scale, rows, rows)
+        if rope_base:
+            # R^T at the sampled positions: embed the rows at their positions of a zero slice
+            full = np.zeros((2, L, d))
+            full[0, rows], full[1, rows] = rdq, rdk
+            un = rope.rope_unrotate(full[:, :, None], rope_base)[:, :, 0]
+            rdq, rdk = un[0, rows], un[1, rows]
         acc["o"][0].append(o[b, rows, h]); acc["o"][1].append(ro)
         acc["lse"][0].append(lse[b, h, rows]); acc["lse"][1].append(rlse)
         acc["dq"][0].append(dq[b, rows, h]); acc["dq"][1].append(rdq)

@@ -76,3 +76,27 @@ def test_host_validation_before_launch(lib):
                          None) == lib.DD_ERR_INVALID_ARG                         # null dO
     assert L.dd_attn_bwd(ctypes.byref(d), *good[:3], good[3], good[3], good[4], *good[:3], 0x100000, 256,
                          None) == lib.DD_ERR_WORKSPACE                           # bwd needs more than the status
+
+
+def test_rope_descriptor_and_workspace(lib):
+    """RoPE adds a [L, d/2] (cos, sin) fp32 table to the backward workspace;
+    a negative or non-finite base is rejected."""
+    plain = lib.make_desc(3, 200, 2, 128)
+    roped = lib.make_desc(3, 200, 2, 128, rope_base=1e4)
+    tab = (200 * 64 * 8 + 255) // 256 * 256
+    assert lib.workspace_size(roped, True) == lib.workspace_size(plain, True) + tab
+    assert lib.workspace_size(roped, False) == 256
+    for bad in (-1.0, float("nan"), float("inf")):
+        assert lib.workspace_size(lib.make_desc(3, 200, 2, 128, rope_base=bad), True) == 0
+
+
+def test_rope_qk_host_validation(lib):
+    L = lib.lib()
+    p = [0x10000, 0x20000, 0x30000, 0x40000]
+    call = lambda desc, ptrs: L.dd_rope_qk(ctypes.byref(desc), *ptrs, None)
+    d = lib.make_desc(2, 256, 2, 128, rope_base=1e4)
+    assert call(lib.make_desc(2, 256, 2, 128), p) == lib.DD_ERR_INVALID_ARG        # rope_base = 0
+    assert call(d, [None] + p[1:]) == lib.DD_ERR_INVALID_ARG                      # null q
+    assert call(d, p[:3] + [0x40004]) == lib.DD_ERR_INVALID_ARG                   # misaligned k_rot
+    assert call(lib.make_desc(2, 256, 2, 80, rope_base=1e4), p) == lib.DD_ERR_UNSUPPORTED
+    assert L.dd_rope_qk(None, *p, None) == lib.DD_ERR_INVALID_ARG
