@@ -87,8 +87,9 @@ typedef struct {
 /* Workspace bytes for dd_attn_fwd (for_bwd = 0) or dd_attn_bwd (for_bwd = 1):
  * the status word, and for bwd the fp32 dQ accumulator (B*H*L128*d floats) plus
  * the per-row D_i and LSE_i*log2(e) vectors [B, H, L128], L128 = L rounded up
- * to a multiple of 128, plus, when rope_base > 0, a [L, d/2] table of
- * (cos, sin) pairs (fp32). Returns 0 for an invalid descriptor. */
+ * to a multiple of 128, plus, when rope_base > 0, two copies of the
+ * (cos, sin) table of every position and pair (fp32, (L rounded up to 32 +
+ * L) * d/2 pairs). Returns 0 for an invalid descriptor. */
 size_t dd_attn_workspace_size(const dd_attn_desc* desc, int for_bwd);
 
 /* Forward (Sec. 2.2 step; mask per cu_doc_offsets): writes o and lse. */

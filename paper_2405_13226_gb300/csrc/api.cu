@@ -54,6 +54,9 @@ size_t bwd_acc_bytes(const dd_attn_desc* d) {
   return align256((size_t)d->B * d->H * round128(d->L) * d->d * sizeof(float));
 }
 size_t rope_tab_bytes(const dd_attn_desc* d) {
+  return has_rope(d) ? align256((size_t)((d->L + 31) / 32 * 32) * (d->d / 2) * sizeof(float2)) : 0;
+}
+size_t rope_rows_bytes(const dd_attn_desc* d) {
   return has_rope(d) ? align256((size_t)d->L * (d->d / 2) * sizeof(float2)) : 0;
 }
 
@@ -140,7 +143,7 @@ extern "C" {
 size_t dd_attn_workspace_size(const dd_attn_desc* desc, int for_bwd) {
   if (check_desc(desc) != DD_OK) return 0;
   if (!for_bwd) return kStatusBytes;
-  return kStatusBytes + 2 * bwd_vec_bytes(desc) + bwd_acc_bytes(desc) + rope_tab_bytes(desc);
+  return kStatusBytes + 2 * bwd_vec_bytes(desc) + bwd_acc_bytes(desc) + rope_tab_bytes(desc) + rope_rows_bytes(desc);
 }
 
 dd_status dd_rope_qk(const dd_attn_desc* desc, const void* q, const void* k, void* q_rot, void* k_rot,
@@ -237,9 +240,9 @@ dd_status dd_attn_bwd_phases(const dd_attn_desc* desc, const void* q, const void
   p.dq = static_cast<__nv_bfloat16*>(dq);
   p.dk = static_cast<__nv_bfloat16*>(dk);
   p.dv = static_cast<__nv_bfloat16*>(dv);
-  p.rope_tab = has_rope(desc) ? reinterpret_cast<float2*>(w + kStatusBytes + 2 * bwd_vec_bytes(desc) +
-                                                           bwd_acc_bytes(desc))
-                              : nullptr;
+  uint8_t* rope_base = w + kStatusBytes + 2 * bwd_vec_bytes(desc) + bwd_acc_bytes(desc);
+  p.rope_tab = has_rope(desc) ? reinterpret_cast<float4*>(rope_base) : nullptr;
+  p.rope_tab_rows = has_rope(desc) ? reinterpret_cast<float2*>(rope_base + rope_tab_bytes(desc)) : nullptr;
   p.rope = has_rope(desc) ? rope_freq(desc) : RopeFreq{};
   p.status = static_cast<int*>(ws);
   p.timeout_ns = wait_limit_ns();

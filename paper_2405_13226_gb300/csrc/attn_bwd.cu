@@ -151,7 +151,7 @@ __global__ void __launch_bounds__(256) attn_bwd_post_kernel(const BwdParams p) {
     float f[8] = {x.x * p.scale, x.y * p.scale, x.z * p.scale, x.w * p.scale,
                   y.x * p.scale, y.y * p.scale, y.z * p.scale, y.w * p.scale};
     if (p.rope_tab) {  // dq = R^T dq_rot: pairs j = 4 part .. 4 part + 3 at position i
-      const float4* t4 = reinterpret_cast<const float4*>(p.rope_tab + (long long)i * (D / 2) + part * 4);
+      const float4* t4 = reinterpret_cast<const float4*>(p.rope_tab_rows + (long long)i * (D / 2) + part * 4);
       const float4 a = t4[0], c = t4[1];
       rope_unrotate_pair(f[0], f[1], a.x, a.y);
       rope_unrotate_pair(f[2], f[3], a.z, a.w);
@@ -481,7 +481,7 @@ __global__ void __launch_bounds__(320, 1)
         uint32_t v[32];
         tmem_ld32(tl + C::TM_DK + c * 32, v);
         tmem_ld_wait(v);
-        if (kv < p.L) store_dk_row32(dst + c * 32, v, p.scale, p.rope_tab, kv, D / 2, c * 16);
+        if (kv < p.L) store_dk_row32(dst + c * 32, v, p.scale, p.rope_tab, kv, D, c * 8);
       }
     }
   }
@@ -516,7 +516,8 @@ static cudaError_t launch_bwd_d(const CUtensorMap& tq, const CUtensorMap& tk, co
   const int ew_blocks = (int)std::min<long long>((work + 255) / 256, (long long)nsm * 8);
   cudaError_t e = cudaSuccess;
   if (phases & 1) {
-    if (p.rope_tab && (e = launch_rope_table(p.L, D, p.rope, p.rope_tab, stream)) != cudaSuccess) return e;
+    if (p.rope_tab && (e = launch_rope_table(p.L, D, p.rope, p.rope_tab, p.rope_tab_rows, stream)) != cudaSuccess)
+      return e;
     attn_bwd_pre_kernel<D><<<ew_blocks, 256, 0, stream>>>(p);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }

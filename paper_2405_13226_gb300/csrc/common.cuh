@@ -82,6 +82,14 @@ __device__ __forceinline__ float2 rope_cos_sin(int m, float hi, float lo) {
   return make_float2(fmaf(-e, s, fmaf(-h, c, c)), fmaf(e, c, fmaf(-h, s, s)));
 }
 
+// The backward's (cos, sin) table: one float4 (cos, sin of pair 2jj, cos, sin
+// of pair 2jj + 1) per (position m, pair-pair jj), laid out
+// [ceil(L/32)][d/4][32 positions] so that the 32 lanes of a warp, holding 32
+// consecutive positions, read one contiguous 512-byte run for a given jj.
+__device__ __forceinline__ long long rope_tab_index(int m, int d, int jj) {
+  return ((long long)(m >> 5) * (d / 4) + jj) * 32 + (m & 31);
+}
+
 // g <- R^T g for one rotated pair (cs = (cos, sin)).
 __device__ __forceinline__ void rope_unrotate_pair(float& g0, float& g1, float c, float s) {
   const float a = fmaf(g0, c, g1 * s);
@@ -90,27 +98,31 @@ __device__ __forceinline__ void rope_unrotate_pair(float& g0, float& g1, float c
   g1 = b;
 }
 
-// One 32-column slice of a dK row: dk = scale * acc, then R^T at position m
-// when tab != nullptr (pairs j0 .. j0 + 15 of a row of `half` table entries).
-__device__ __forceinline__ void store_dk_row32(__nv_bfloat16* dst, const uint32_t (&v)[32], float sc,
-                                               const float2* tab, int m, int half, int j0) {
-  float f[32];
-#pragma unroll
-  for (int e = 0; e < 32; e++) f[e] = __uint_as_float(v[e]) * sc;
-  if (tab) {
-    const float4* t4 = reinterpret_cast<const float4*>(tab + (long long)m * half + j0);
-#pragma unroll
-    for (int u = 0; u < 8; u++) {
-      const float4 cs = t4[u];
-      rope_unrotate_pair(f[4 * u], f[4 * u + 1], cs.x, cs.y);
-      rope_unrotate_pair(f[4 * u + 2], f[4 * u + 3], cs.z, cs.w);
-    }
-  }
+// 32 fp32 values -> 32 bf16 at dst (16-byte aligned).
+__device__ __forceinline__ void store_row32(__nv_bfloat16* dst, const float (&f)[32]) {
   uint4* d4 = reinterpret_cast<uint4*>(dst);
 #pragma unroll
   for (int q = 0; q < 4; q++)
     d4[q] = make_uint4(pack_bf16x2(f[8 * q], f[8 * q + 1]), pack_bf16x2(f[8 * q + 2], f[8 * q + 3]),
                        pack_bf16x2(f[8 * q + 4], f[8 * q + 5]), pack_bf16x2(f[8 * q + 6], f[8 * q + 7]));
+}
+
+// One 32-column slice of a dK row: dk = scale * acc, then R^T at position m
+// when tab != nullptr (pair-pairs jj0 .. jj0 + 7 of the table above).
+__device__ __forceinline__ void store_dk_row32(__nv_bfloat16* dst, const uint32_t (&v)[32], float sc,
+                                               const float4* tab, int m, int d, int jj0) {
+  float f[32];
+#pragma unroll
+  for (int e = 0; e < 32; e++) f[e] = __uint_as_float(v[e]) * sc;
+  if (tab) {
+#pragma unroll
+    for (int u = 0; u < 8; u++) {
+      const float4 cs = tab[rope_tab_index(m, d, jj0 + u)];
+      rope_unrotate_pair(f[4 * u], f[4 * u + 1], cs.x, cs.y);
+      rope_unrotate_pair(f[4 * u + 2], f[4 * u + 3], cs.z, cs.w);
+    }
+  }
+  store_row32(dst, f);
 }
 
 struct FwdParams {
@@ -138,7 +150,8 @@ struct BwdParams {
   __nv_bfloat16* dq;
   __nv_bfloat16* dk;
   __nv_bfloat16* dv;
-  float2* rope_tab;  // [L, d/2] (cos, sin) of m theta_j, or nullptr without RoPE
+  float4* rope_tab;       // (cos, sin) of m theta_j (layout of rope_tab_index), or nullptr without RoPE
+  float2* rope_tab_rows;  // the same values row-major [L, d/2] (read by the dq post kernel)
   RopeFreq rope;     // frequencies that fill rope_tab
   int* status;
   unsigned long long timeout_ns;
@@ -162,6 +175,6 @@ cudaError_t launch_attn_bwd_main_d128(const CUtensorMap& tq, const CUtensorMap& 
 cudaError_t launch_attn_bwd(int d, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
                             const CUtensorMap& tdo, const BwdParams& p, int phases, cudaStream_t stream);
 cudaError_t launch_rope_qk(const RopeParams& p, cudaStream_t stream);
-cudaError_t launch_rope_table(int L, int d, const RopeFreq& f, float2* tab, cudaStream_t stream);
+cudaError_t launch_rope_table(int L, int d, const RopeFreq& f, float4* tab, float2* tab_rows, cudaStream_t stream);
 
 }  // namespace ddattn

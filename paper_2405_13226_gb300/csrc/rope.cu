@@ -1,6 +1,6 @@
 // Rotary position embedding of q and k (consecutive component pairs rotated by
 // m * f_b^(-2j/d), m = position inside the sequence), and the (cos, sin) table
-// the backward uses to rotate dq and dk back.
+// the backward uses to rotate dq and dk back (layout of rope_tab_index).
 //
 // rope_qk_kernel is bound by HBM: it reads q and k once and writes q_rot and
 // k_rot once (4 * B*L*H*d*2 bytes). A CTA takes kRows consecutive token rows:
@@ -43,7 +43,7 @@ __global__ void __launch_bounds__(kThreads) rope_qk_kernel(const __grid_constant
         const bool is_k = t >= per_tensor;
         const int idx = is_k ? t - per_tensor : t;
         const uint4* src = reinterpret_cast<const uint4*>((is_k ? p.k : p.q) + base) + idx;
-        x[u] = *src;
+        x[u] = __ldcs(src);   // read once: streaming
       }
     }
 #pragma unroll
@@ -63,18 +63,24 @@ __global__ void __launch_bounds__(kThreads) rope_qk_kernel(const __grid_constant
           w[e] = pack_bf16x2(fmaf(v.x, r.x, -v.y * r.y), fmaf(v.x, r.y, v.y * r.x));
         }
         uint4* dst = reinterpret_cast<uint4*>((is_k ? p.k_rot : p.q_rot) + base) + idx;
-        *dst = make_uint4(w[0], w[1], w[2], w[3]);
+        __stcs(dst, make_uint4(w[0], w[1], w[2], w[3]));
       }
     }
   }
 }
 
-__global__ void __launch_bounds__(256) rope_table_kernel(int L, int half, const __grid_constant__ RopeFreq f,
-                                                         float2* tab) {
-  const long long n = (long long)L * half;
+// One thread per (position m, pair-pair jj): two (cos, sin) values into the
+// float4 of rope_tab_index(m, d, jj) and into the row-major copy.
+__global__ void __launch_bounds__(256) rope_table_kernel(int L, int d, const __grid_constant__ RopeFreq f,
+                                                         float4* tab, float2* tab_rows) {
+  const int quarter = d / 4;
+  const long long n = (long long)L * quarter;
   for (long long t = (long long)blockIdx.x * blockDim.x + threadIdx.x; t < n; t += (long long)gridDim.x * blockDim.x) {
-    const int m = (int)(t / half), j = (int)(t % half);
-    tab[t] = rope_cos_sin(m, f.hi[j], f.lo[j]);
+    const int m = (int)(t / quarter), jj = (int)(t % quarter);
+    const float2 a = rope_cos_sin(m, f.hi[2 * jj], f.lo[2 * jj]);
+    const float2 b = rope_cos_sin(m, f.hi[2 * jj + 1], f.lo[2 * jj + 1]);
+    tab[rope_tab_index(m, d, jj)] = make_float4(a.x, a.y, b.x, b.y);
+    reinterpret_cast<float4*>(tab_rows)[t] = make_float4(a.x, a.y, b.x, b.y);  // = [m][2jj], [m][2jj+1]
   }
 }
 
@@ -85,10 +91,10 @@ cudaError_t launch_rope_qk(const RopeParams& p, cudaStream_t stream) {
   return cudaGetLastError();
 }
 
-cudaError_t launch_rope_table(int L, int d, const RopeFreq& f, float2* tab, cudaStream_t stream) {
-  const long long n = (long long)L * (d / 2);
+cudaError_t launch_rope_table(int L, int d, const RopeFreq& f, float4* tab, float2* tab_rows, cudaStream_t stream) {
+  const long long n = (long long)L * (d / 4);
   const int blocks = (int)std::min<long long>((n + 255) / 256, 4096);
-  rope_table_kernel<<<blocks, 256, 0, stream>>>(L, d / 2, f, tab);
+  rope_table_kernel<<<blocks, 256, 0, stream>>>(L, d, f, tab, tab_rows);
   return cudaGetLastError();
 }
 

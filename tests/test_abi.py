@@ -79,11 +79,12 @@ def test_host_validation_before_launch(lib):
 
 
 def test_rope_descriptor_and_workspace(lib):
-    """RoPE adds a [L, d/2] (cos, sin) fp32 table to the backward workspace;
+    """RoPE adds two copies of the (cos, sin) fp32 table to the backward workspace;
     a negative or non-finite base is rejected."""
     plain = lib.make_desc(3, 200, 2, 128)
     roped = lib.make_desc(3, 200, 2, 128, rope_base=1e4)
-    tab = (200 * 64 * 8 + 255) // 256 * 256
+    tab = (224 * 64 * 8 + 255) // 256 * 256        # warp-blocked layout, positions rounded up to 32
+    tab += (200 * 64 * 8 + 255) // 256 * 256       # row-major copy
     assert lib.workspace_size(roped, True) == lib.workspace_size(plain, True) + tab
     assert lib.workspace_size(roped, False) == 256
     for bad in (-1.0, float("nan"), float("inf")):
