@@ -367,35 +367,20 @@ __global__ void __launch_bounds__(512, 1)
       fence_proxy_async_smem();
       mbar_arrive(&bars->dss_full);
     }
-    // Epilogue: dK rows, columns [qh, qh + 64), scaled (and rotated back with
-    // RoPE). These warps wait here while the last MMAs run, so the row's
-    // (cos, sin) pairs are fetched before the wait and their latency is hidden.
-    float4 cs[16];
-    const bool rope = p.rope_tab != nullptr && kv < p.L;
-    if (rope) {
-#pragma unroll
-      for (int u = 0; u < 16; u++) cs[u] = p.rope_tab[rope_tab_index(kv, D, qh / 4 + u)];
-    }
+    // Epilogue: dV rows.
     if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&bars->mma_done, 0, wd));
     if (ok) {
       tc_fence_after();
-      __nv_bfloat16* dst = p.dk + ((seq0 + kvc) * p.H + h) * D + qh;
-#pragma unroll
+      __nv_bfloat16* dst = p.dv + ((seq0 + kvc) * p.H + h) * D + qh;
+#pragma unroll 1
       for (int c = 0; c < 2; c++) {
         uint32_t v[32];
-        tmem_ld32(tl + C::TM_DK + qh + c * 32, v);
+        tmem_ld32(tl + C::TM_DV + qh + c * 32, v);
         tmem_ld_wait(v);
         if (kv < p.L) {
           float f[32];
 #pragma unroll
-          for (int e = 0; e < 32; e++) f[e] = __uint_as_float(v[e]) * p.scale;
-          if (rope) {
-#pragma unroll
-            for (int u = 0; u < 8; u++) {
-              rope_unrotate_pair(f[4 * u], f[4 * u + 1], cs[8 * c + u].x, cs[8 * c + u].y);
-              rope_unrotate_pair(f[4 * u + 2], f[4 * u + 3], cs[8 * c + u].z, cs[8 * c + u].w);
-            }
-          }
+          for (int e = 0; e < 32; e++) f[e] = __uint_as_float(v[e]);
           store_row32(dst + c * 32, f);
         }
       }
@@ -436,24 +421,20 @@ __global__ void __launch_bounds__(512, 1)
       }
     }
     if (lane == 0) bulk_wait<0>();
-    // Epilogue: dV rows.
+    // Epilogue: dK rows (scaled; rotated back with RoPE).
     if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&bars->mma_done, 0, wd));
     if (ok) {
       tc_fence_after();
       const int kv = kv0 + t;
       const int kvc = kv < p.L ? kv : p.L - 1;
-      __nv_bfloat16* dst = p.dv + ((seq0 + kvc) * p.H + h) * D;
+      __nv_bfloat16* dst = p.dk + ((seq0 + kvc) * p.H + h) * D;
 #pragma unroll 1
       for (int c = 0; c < D / 32; c++) {
         uint32_t v[32];
-        tmem_ld32(tl + C::TM_DV + c * 32, v);
+        tmem_ld32(tl + C::TM_DK + c * 32, v);
         tmem_ld_wait(v);
-        if (kv < p.L) {
-          float f[32];
-#pragma unroll
-          for (int e = 0; e < 32; e++) f[e] = __uint_as_float(v[e]);
-          store_row32(dst + c * 32, f);
-        }
+        // With RoPE, R^T per pair from the warp-coalesced (cos, sin) table.
+        if (kv < p.L) store_dk_row32(dst + c * 32, v, p.scale, p.rope_tab, kv, D, c * 8);
       }
     }
   }
