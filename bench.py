@@ -251,9 +251,13 @@ def run_ours(args):
     # inputs: [T, H, D] bf16 per tensor (256 MiB each, larger than L2), seeded
     qb, kb, vb, gb = wl.attn_inputs(1, T, H, D, seed=rank)
     q, k, v, g = (to_dev(x, dev) for x in (qb, kb, vb, gb))
-    ws = ddattn.new_workspace(ddattn.make_desc(1, T, H, D), dev)   # same size for every bucket
     sweep = [args.only_L] if args.only_L else list(wl.BUCKETS)
-    buckets = [Bucket(ddattn, q, k, v, g, T // L, L, H, ws=ws) for L in sweep]
+    rb = args.rope_base
+    # one workspace sized for the largest bucket (RoPE tables grow with L)
+    ws = ddattn.new_workspace(max((ddattn.make_desc(T // L, L, H, D, None, None, rb) for L in sweep),
+                                  key=ddattn.workspace_size), dev)
+    qk_rot = (torch.empty_like(q), torch.empty_like(k)) if rb else None
+    buckets = [Bucket(ddattn, q, k, v, g, T // L, L, H, ws=ws, rope_base=rb, qk_rot=qk_rot) for L in sweep]
     for bk in buckets:   # one correctness-agnostic pass so every instance is loaded
         bk.fwd(stream); bk.bwd(stream)
     torch.cuda.synchronize()
@@ -340,7 +344,7 @@ def run_ours(args):
         "dtype": "bf16 in, fp32 accumulate", "data": "synthetic (seeded N(0,1) bf16 q,k,v,dO)",
         "config": {"workload": "bucket sweep L=256..8192, 65536 tokens per call, H=16, d=128, causal; "
                                "step = fwd+bwd of every bucket (6 calls)",
-                   "tokens_per_call": T, "H": H, "d": D, "buckets": sweep,
+                   "tokens_per_call": T, "H": H, "d": D, "buckets": sweep, "rope_base": args.rope_base,
                    "l2": "inputs larger than L2 (4 x 256 MiB bf16 tensors)", "parallelism": "replicas" if world > 1 else "1 GPU"},
         "ms_per_64k_token_step_by_bucket": {str(p["L"]): p["ms"] for p in per_bucket},
         "per_bucket": per_bucket,
@@ -573,6 +577,8 @@ def main():
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end measurement")
     ap.add_argument("--only-L", type=int, default=0, help="run one bucket of the sweep (profiling)")
+    ap.add_argument("--rope-base", type=float, default=0.0,
+                    help="run the headline step with RoPE of this base frequency (rotation + fwd + bwd)")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
