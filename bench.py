@@ -6,7 +6,8 @@ of one 65536-token batch of every bucket (6 calls of each). `value` is the
 algorithmic TFLOP/s over the step (14 d H sum_seq L(L+1)/2 flops per call).
 Also reported: per-bucket ms and TFLOP/s, the document-masked 8x8192
 concat-and-chunk step (16 seeds), the Pack-8k+DM step, an Algorithm 1
-stream (Grow-P2, 8 cycles), the sweep with RoPE (f_b = 100k), the
+stream (Grow-P2, 8 cycles) and every Table 2 curriculum, the sweep with RoPE
+(f_b = 100k), the 3B (H=32, d=80) and 7B (H=32, d=128) head shapes, the
 long-context bucket (B=4, L=16384, H=32), the roofline of the dominant kernel,
 an end-to-end number through host buffers, and the fp64 oracle's throughput on
 this host's cores.
@@ -204,12 +205,12 @@ def to_dev(bits, dev):
 class Bucket:
     """Buffers of one call shape; inputs are views of shared [T, H, D] tensors."""
 
-    def __init__(self, ddattn, q, k, v, g, B, L, Hh, offsets=None, ws=None, rope_base=0.0, qk_rot=None):
+    def __init__(self, ddattn, q, k, v, g, B, L, Hh, offsets=None, ws=None, rope_base=0.0, qk_rot=None, Dh=D):
         import torch
         self.dd = ddattn
         self.B, self.L = B, L
         self.rope_base = rope_base
-        shape = (B, L, Hh, D)
+        shape = (B, L, Hh, Dh)
         self.q, self.k, self.v, self.g = (x.view(shape) for x in (q, k, v, g))
         if rope_base:
             # the attention reads the rotated q, k (written by rope_qk each step)
@@ -219,10 +220,10 @@ class Bucket:
         self.lse = torch.empty((B, Hh, L), dtype=torch.float32, device=q.device)
         self.dq, self.dk, self.dv = (torch.empty_like(self.q) for _ in range(3))
         self.off = offsets
-        self.desc = ddattn.make_desc(B, L, Hh, D, None, offsets, rope_base)
+        self.desc = ddattn.make_desc(B, L, Hh, Dh, None, offsets, rope_base)
         self.ws = ws if ws is not None else ddattn.new_workspace(self.desc, q.device)
-        self.flops = wl.attn_flops(B, L, Hh, D, None if offsets is None else offsets.cpu().numpy())
-        self.flops_fwd = wl.attn_flops(B, L, Hh, D, None if offsets is None else offsets.cpu().numpy(), bwd=False)
+        self.flops = wl.attn_flops(B, L, Hh, Dh, None if offsets is None else offsets.cpu().numpy())
+        self.flops_fwd = wl.attn_flops(B, L, Hh, Dh, None if offsets is None else offsets.cpu().numpy(), bwd=False)
         self.flops_bwd = self.flops - self.flops_fwd
 
     def rope(self, stream):
@@ -413,6 +414,25 @@ def extra_workloads(ddattn, q, k, v, g, buckets, ws, stream, peaks, dev):
                                      % len(stream_L),
                          "bucket_steps": {str(L): stream_L.count(L) for L in sorted(sched)},
                          "ms_per_step_mean": cur_ms, "tflops": cur_flops / (cur_ms * 1e-3) / 1e12}
+    # every curriculum of Table 2 with 1 and 8 cycles: each consumes the same bucket steps,
+    # so the expected ms per step is fixed by the per-bucket times; measured = the stream run
+    # in its own order
+    per_L_ms = {bk.L: time_calls(lambda bk=bk: (bk.fwd(stream), bk.bwd(stream)), 5, 1, stream) for bk in buckets}
+    expected = sum(per_L_ms[L] * stream_L.count(L) for L in set(stream_L)) / len(stream_L)
+    curricula = {}
+    for name, odds in wl.CURRICULA.items():
+        for cyc in (1, 8):
+            sl = wl.length_curriculum(sched, dict(zip(wl.BUCKETS, odds)), cyc, T, seed=0)
+            torch.cuda.synchronize()
+            s.record(stream)
+            for L in sl:
+                by_L[L].fwd(stream)
+                by_L[L].bwd(stream)
+            e.record(stream)
+            torch.cuda.synchronize()
+            curricula["%s/%d" % (name, cyc)] = {"measured_ms_per_step": s.elapsed_time(e) / len(sl),
+                                                "first_8_L": sl[:8]}
+    out["curricula"] = {"steps": len(stream_L), "expected_ms_per_step": expected, "per_curriculum": curricula}
     out["dd_vs_dm_step_time_ratio"] = cur_ms / dm_mean
     out["dd_vs_dm_flop_ratio"] = cur_flops / float(np.mean([
         wl.attn_flops(8, 8192, H, D, wl.concat_and_chunk_offsets(sd)) for sd in range(16)]))
@@ -453,6 +473,28 @@ def extra_workloads(ddattn, q, k, v, g, buckets, ws, stream, peaks, dev):
                          / peaks["hbm_gbs"],
                          "per_bucket": rope_rows}
     del qr, kr, rws
+    # other model shapes of the Appendix model table at 65536 tokens per call:
+    # 3B heads (H=32, d=2560/32=80) and 7B heads (H=32, d=4096/32=128)
+    shapes = {}
+    for name, Hh, Dh in (("3B", 32, 80), ("7B", 32, 128)):
+        gen = torch.Generator(device=dev).manual_seed(Dh)
+        xs = [torch.randn(T * Hh * Dh, device=dev, generator=gen).to(torch.bfloat16) for _ in range(4)]
+        sws = ddattn.new_workspace(ddattn.make_desc(1, T, Hh, Dh), dev)
+        rows = []
+        for L in wl.BUCKETS:
+            bk = Bucket(ddattn, *xs, T // L, L, Hh, ws=sws, Dh=Dh)
+            ms = time_calls(lambda: (bk.fwd(stream), bk.bwd(stream)), 3, 1, stream)
+            rows.append({"L": L, "ms": ms, "tflops": bk.flops / (ms * 1e-3) / 1e12})
+        st = ddattn.poll_status(sws)
+        if st != 0:
+            raise RuntimeError("device status %d (%s)" % (st, ddattn.status_string(st)))
+        shapes[name] = {"H": Hh, "d": Dh, "ms_per_step": sum(x["ms"] for x in rows),
+                        "tflops": sum(wl.attn_flops(T // x["L"], x["L"], Hh, Dh) for x in rows)
+                        / (sum(x["ms"] for x in rows) * 1e-3) / 1e12, "per_bucket": rows}
+        del xs, sws
+    torch.cuda.empty_cache()
+    out["model_shapes"] = {"workload": "bucket sweep at 65536 tokens per call, inputs N(0,1) bf16 from a seeded "
+                                       "torch generator", **shapes}
     # long-context bucket: B=4, L=16384, H=32, q/k x3
     qb, kb, vb, gb = wl.attn_inputs(4, 16384, 32, D, seed=0, qk_mult=3.0)
     lq, lk, lv, lg = (to_dev(x, dev) for x in (qb, kb, vb, gb))

@@ -67,7 +67,7 @@ extern "C" {
 typedef enum {
   DD_OK = 0,
   DD_ERR_INVALID_ARG = 1,     /* null / misaligned pointer, bad sizes */
-  DD_ERR_UNSUPPORTED = 2,     /* head dim other than 64 or 128, device not sm_103 */
+  DD_ERR_UNSUPPORTED = 2,     /* head dim other than 64, 80 or 128, device not sm_103 */
   DD_ERR_WORKSPACE = 3,       /* workspace missing or smaller than required */
   DD_ERR_CUDA = 4,            /* a CUDA runtime call or launch failed */
   DD_ERR_DEVICE_TIMEOUT = 5   /* a bounded device-side wait expired */
@@ -77,7 +77,7 @@ typedef struct {
   int32_t B;                       /* sequences per call (>= 1) */
   int32_t L;                       /* tokens per sequence (>= 1; multiples of 128 are the fast path) */
   int32_t H;                       /* heads (>= 1) */
-  int32_t d;                       /* head dim: 64 or 128 */
+  int32_t d;                       /* head dim: 64, 80 (OpenLM-3B heads) or 128 */
   float scale;                     /* softmax scale, usually 1/sqrt(d); finite */
   const int32_t* cu_doc_offsets;   /* DEVICE pointer or NULL (plain causal) */
   int32_t n_offsets;               /* entries of cu_doc_offsets (>= 2 when non-NULL) */
@@ -85,7 +85,8 @@ typedef struct {
 } dd_attn_desc;
 
 /* Workspace bytes for dd_attn_fwd (for_bwd = 0) or dd_attn_bwd (for_bwd = 1):
- * the status word, and for bwd the fp32 dQ accumulator (B*H*L128*d floats) plus
+ * the status word, and for bwd the fp32 dQ accumulator (B*H*L128*d' floats,
+ * d' = 64 for d = 64, else d rounded up to a multiple of 32) plus
  * the per-row D_i and LSE_i*log2(e) vectors [B, H, L128], L128 = L rounded up
  * to a multiple of 128, plus, when rope_base > 0, two copies of the
  * (cos, sin) table of every position and pair (fp32, (L rounded up to 32 +

@@ -23,7 +23,7 @@ dd_status check_desc(const dd_attn_desc* d) {
   if (!d) return DD_ERR_INVALID_ARG;
   if (d->B < 1 || d->L < 1 || d->H < 1) return DD_ERR_INVALID_ARG;
   if (d->B > 65535 || d->H > 65535) return DD_ERR_INVALID_ARG;  // grid y/z limits
-  if (d->d != 64 && d->d != 128) return DD_ERR_UNSUPPORTED;
+  if (d->d != 64 && d->d != 80 && d->d != 128) return DD_ERR_UNSUPPORTED;
   if (!std::isfinite(d->scale) || !(d->scale > 0.f)) return DD_ERR_INVALID_ARG;
   if (d->cu_doc_offsets) {
     if (d->n_offsets < 2 || (reinterpret_cast<uintptr_t>(d->cu_doc_offsets) & 3u)) return DD_ERR_INVALID_ARG;
@@ -50,8 +50,10 @@ RopeFreq rope_freq(const dd_attn_desc* d) {
 size_t bwd_vec_bytes(const dd_attn_desc* d) {
   return align256((size_t)d->B * d->H * round128(d->L) * sizeof(float));
 }
+// fp32 dQ accumulator: [B, H, L128, 64] for d = 64, [B, H, ceil(d/32), L128, 32] otherwise.
 size_t bwd_acc_bytes(const dd_attn_desc* d) {
-  return align256((size_t)d->B * d->H * round128(d->L) * d->d * sizeof(float));
+  const size_t cols = d->d == 64 ? 64 : (size_t)(d->d + 31) / 32 * 32;
+  return align256((size_t)d->B * d->H * round128(d->L) * cols * sizeof(float));
 }
 size_t rope_tab_bytes(const dd_attn_desc* d) {
   return has_rope(d) ? align256((size_t)((d->L + 31) / 32 * 32) * (d->d / 2) * sizeof(float2)) : 0;
@@ -276,7 +278,7 @@ const char* dd_status_string(dd_status s) {
   switch (s) {
     case DD_OK: return "ok";
     case DD_ERR_INVALID_ARG: return "invalid argument";
-    case DD_ERR_UNSUPPORTED: return "unsupported (head dim must be 64 or 128; device must be sm_103)";
+    case DD_ERR_UNSUPPORTED: return "unsupported (head dim must be 64, 80 or 128; device must be sm_103)";
     case DD_ERR_WORKSPACE: return "workspace missing, misaligned or too small";
     case DD_ERR_CUDA: return "CUDA runtime error";
     case DD_ERR_DEVICE_TIMEOUT: return "device-side wait timed out";

@@ -72,11 +72,19 @@ struct BwdBars {
 };
 static_assert(sizeof(BwdBars) <= 256, "barrier block");
 
+// Columns of one row of the fp32 dQ accumulator: d = 64 keeps [.., L128, 64];
+// the d = 80 / 128 kernel uses ceil(d/32) chunks of 32 columns.
+template <int D>
+__host__ __device__ constexpr int acc_cols() { return D == 64 ? 64 : (D + 31) / 32 * 32; }
+
 // ------------------------------------------------------------------ pre
-// One group of d/8 threads per (b, i, h) row, rows in memory order.
+// One group of G threads per (b, i, h) row, rows in memory order; the first
+// d/8 threads of a group load 8 bf16 each (G = d/8 rounded up to a power of
+// two, the shuffle width).
 template <int D>
 __global__ void __launch_bounds__(256) attn_bwd_pre_kernel(const BwdParams p) {
-  constexpr int G = D / 8;  // threads per row, 8 bf16 each
+  constexpr int NP = D / 8;                                        // 16-byte parts per row
+  constexpr int G = NP <= 8 ? 8 : (NP <= 16 ? 16 : 32);            // threads per row
   const long long nrows = (long long)p.B * p.L * p.H;
   const long long total = nrows * G;
   const long long tid = (long long)blockIdx.x * blockDim.x + threadIdx.x;
@@ -89,7 +97,7 @@ __global__ void __launch_bounds__(256) attn_bwd_pre_kernel(const BwdParams p) {
     const long long row = valid ? t / G : 0;
     const int part = (int)(t % G);
     float acc = 0.f;
-    if (valid) {
+    if (valid && part < NP) {
       const uint4 a = reinterpret_cast<const uint4*>(p.o + row * D)[part];
       const uint4 g = reinterpret_cast<const uint4*>(p.dO + row * D)[part];
       const __nv_bfloat162* a2 = reinterpret_cast<const __nv_bfloat162*>(&a);
@@ -124,7 +132,7 @@ __global__ void __launch_bounds__(256) attn_bwd_pre_kernel(const BwdParams p) {
     p.lse2_pad[o] = INFINITY;
   }
   // zero the dQ accumulator
-  const long long n4 = (long long)p.B * p.H * p.L128 * D / 4;
+  const long long n4 = (long long)p.B * p.H * p.L128 * acc_cols<D>() / 4;
   float4* acc4 = reinterpret_cast<float4*>(p.dq_acc);
   for (long long t = tid; t < n4; t += stride) acc4[t] = make_float4(0.f, 0.f, 0.f, 0.f);
 }
@@ -142,10 +150,11 @@ __global__ void __launch_bounds__(256) attn_bwd_post_kernel(const BwdParams p) {
     const long long bi = row / p.H;
     const int i = (int)(bi % p.L);
     const int b = (int)(bi / p.L);
-    // d = 64: accumulator rows [B, H, L128, 64]; d = 128: [B, H, 4 chunks, L128, 32]
+    // d = 64: accumulator rows [B, H, L128, 64]; d = 80, 128: [B, H, ceil(d/32) chunks, L128, 32]
+    constexpr int NCH = acc_cols<D>() / 32;
     const long long bh = (long long)b * p.H + h;
-    const float* srcf = (D == 128) ? p.dq_acc + ((bh * 4 + (part >> 2)) * p.L128 + i) * 32 + (part & 3) * 8
-                                   : p.dq_acc + (bh * p.L128 + i) * D + part * 8;
+    const float* srcf = (D != 64) ? p.dq_acc + ((bh * NCH + (part >> 2)) * p.L128 + i) * 32 + (part & 3) * 8
+                                  : p.dq_acc + (bh * p.L128 + i) * D + part * 8;
     const float4* src = reinterpret_cast<const float4*>(srcf);
     const float4 x = src[0], y = src[1];
     float f[8] = {x.x * p.scale, x.y * p.scale, x.z * p.scale, x.w * p.scale,
@@ -481,7 +490,7 @@ __global__ void __launch_bounds__(320, 1)
         uint32_t v[32];
         tmem_ld32(tl + C::TM_DK + c * 32, v);
         tmem_ld_wait(v);
-        if (kv < p.L) store_dk_row32(dst + c * 32, v, p.scale, p.rope_tab, kv, D, c * 8);
+        if (kv < p.L) store_dk_row32(dst + c * 32, v, p.scale, p.rope_tab, kv, D, c * 8, 32);
       }
     }
   }
@@ -498,12 +507,14 @@ template <int D>
 static cudaError_t launch_bwd_d(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
                                 const CUtensorMap& tdo, const BwdParams& p, int phases, cudaStream_t stream) {
   using C = BwdCfg<D>;
-  static bool attr_set = false;
-  if (!attr_set && D != 128) {
-    cudaError_t e =
-        cudaFuncSetAttribute(attn_bwd_main_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_BYTES);
-    if (e != cudaSuccess) return e;
-    attr_set = true;
+  if constexpr (D == 64) {
+    static bool attr_set = false;
+    if (!attr_set) {
+      cudaError_t e =
+          cudaFuncSetAttribute(attn_bwd_main_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_BYTES);
+      if (e != cudaSuccess) return e;
+      attr_set = true;
+    }
   }
   static int nsm = 0;
   if (!nsm) {
@@ -522,8 +533,8 @@ static cudaError_t launch_bwd_d(const CUtensorMap& tq, const CUtensorMap& tk, co
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
   if (phases & 2) {
-    if constexpr (D == 128) {
-      if ((e = launch_attn_bwd_main_d128(tq, tk, tv, tdo, p, stream)) != cudaSuccess) return e;
+    if constexpr (D != 64) {
+      if ((e = launch_attn_bwd_main_d128(D, tq, tk, tv, tdo, p, stream)) != cudaSuccess) return e;
     } else {
       dim3 grid(p.nkt, p.H, p.B);
       attn_bwd_main_kernel<D><<<grid, C::THREADS, C::SMEM_BYTES, stream>>>(tq, tk, tv, tdo, p);
@@ -540,6 +551,7 @@ static cudaError_t launch_bwd_d(const CUtensorMap& tq, const CUtensorMap& tk, co
 cudaError_t launch_attn_bwd(int d, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
                             const CUtensorMap& tdo, const BwdParams& p, int phases, cudaStream_t stream) {
   if (d == 64) return launch_bwd_d<64>(tq, tk, tv, tdo, p, phases, stream);
+  if (d == 80) return launch_bwd_d<80>(tq, tk, tv, tdo, p, phases, stream);
   return launch_bwd_d<128>(tq, tk, tv, tdo, p, phases, stream);
 }
 

@@ -1,4 +1,4 @@
-// Attention backward main kernel for head dim 128 on sm_103a.
+// Attention backward main kernel for head dims 128 and 80 on sm_103a.
 //
 // One CTA per 128-key tile of one (sequence, head), walking the live 128-row
 // query tiles from the diagonal to the end of the tile's last document (the
@@ -38,12 +38,20 @@
 // 128 registers per thread; WG3 gives registers back (setmaxnreg.dec to 56) and
 // the other three groups take them (setmaxnreg.inc to 152): 4*32*56 +
 // 12*32*152 = 65536, exactly the launch's register file share.
+//
+// d = 80 (OpenLM-3B heads) uses the same tiles: each is two 64-column swizzle
+// blocks, the second holding columns 64..79 and TMA zero fill beyond. The
+// contractions over d (S^T, dP^T) take 5 K-steps instead of 8, dV and dK are
+// N = 80 UMMAs, and dQ^T stays M = 128 (its rows 80..127 are zero: K's padded
+// columns), drained by the first three warps into a 3-chunk accumulator.
 #include "common.cuh"
 
 namespace ddattn {
 
-struct Bwd128 {
-  static constexpr int D = 128, BN = 128, BQ = 128;
+template <int D_>
+struct BwdBig {
+  static constexpr int D = D_, BN = 128, BQ = 128;
+  static constexpr int NCH = (D + 31) / 32;              // 32-column chunks of dQ^T / dK / dV
   static constexpr int BLK = 128 * 128;                  // [128 rows][64] bf16, 128B swizzle
   static constexpr int TILE = 2 * BLK;                   // [128 rows][128] bf16
   static constexpr int OFF_K = 0;
@@ -51,7 +59,7 @@ struct Bwd128 {
   static constexpr int OFF_Q = OFF_V + TILE;             // 2 stages
   static constexpr int OFF_DO = OFF_Q + 2 * TILE;        // 2 stages (dO, then dS^T)
   static constexpr int OFF_STG = OFF_DO + 2 * TILE;      // dQ staging quarter
-  static constexpr int STG_BYTES = 32 * D * 4;
+  static constexpr int STG_BYTES = 4 * 32 * 32 * 4;     // one [32 x 32] fp32 slice per drain warp
   static constexpr int OFF_LSE = OFF_STG + STG_BYTES;    // [2][128] fp32
   static constexpr int OFF_DEL = OFF_LSE + 2 * BQ * 4;   // [2][128] fp32
   static constexpr int OFF_BAR = OFF_DEL + 2 * BQ * 4;
@@ -60,7 +68,7 @@ struct Bwd128 {
   static constexpr int THREADS = 512;
   static constexpr int REGS_LOW = 56, REGS_HIGH = 152;   // setmaxnreg split, see above
 };
-static_assert(4 * 32 * Bwd128::REGS_LOW + 12 * 32 * Bwd128::REGS_HIGH == 512 * 128, "register split");
+static_assert(4 * 32 * BwdBig<128>::REGS_LOW + 12 * 32 * BwdBig<128>::REGS_HIGH == 512 * 128, "register split");
 
 struct Bwd128Bars {
   uint64_t kv_full;
@@ -81,12 +89,14 @@ __device__ __forceinline__ void setmaxnreg_dec() {
   asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(N));
 }
 
+template <int DH>
 __global__ void __launch_bounds__(512, 1)
     attn_bwd_main_d128_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                               const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmDO,
                               const BwdParams p) {
-  using C = Bwd128;
+  using C = BwdBig<DH>;
   constexpr int D = C::D, BQ = C::BQ;
+  constexpr int KD = D / 16;  // K-steps of the contractions over d
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
   Bwd128Bars* bars = reinterpret_cast<Bwd128Bars*>(smem + C::OFF_BAR);
@@ -177,7 +187,7 @@ __global__ void __launch_bounds__(512, 1)
     // ---------------- MMA issuer
     if (lane == 0) {
       constexpr uint32_t id_s = idesc_bf16(128, 128, false, false);  // K / V rows x Q / dO rows (K-major)
-      constexpr uint32_t id_kv = idesc_bf16(128, 128, false, true);  // P^T (TMEM) / dS^T (smem) x dO / Q (MN-major)
+      constexpr uint32_t id_kv = idesc_bf16(128, D, false, true);    // P^T (TMEM) / dS^T (smem) x dO / Q (MN-major)
       constexpr uint32_t id_dq = idesc_bf16(128, 128, true, true);   // K^T (MN-major) x dS^T (MN-major)
       // Descriptors are built once and advanced by adding (byte offset >> 4) to the
       // 14-bit start-address field (all smem offsets here stay below 256 KB).
@@ -192,13 +202,13 @@ __global__ void __launch_bounds__(512, 1)
       if (ok) {
         tc_fence_after();
 #pragma unroll
-        for (int ks = 0; ks < 8; ks++) {  // S^T_0 = K Q_0^T into R[0]
+        for (int ks = 0; ks < KD; ks++) {  // S^T_0 = K Q_0^T into R[0]
           const uint32_t off = ((ks >> 2) * C::BLK + (ks & 3) * 32) >> 4;
           umma_bf16(tmem + C::TM_R, dK_k0 + off, dQ_k0 + off, id_s, ks > 0 ? 1u : 0u);
         }
         umma_commit(&bars->s_full);
 #pragma unroll
-        for (int ks = 0; ks < 8; ks++) {  // dP^T_0 = V dO_0^T into R[1]
+        for (int ks = 0; ks < KD; ks++) {  // dP^T_0 = V dO_0^T into R[1]
           const uint32_t off = ((ks >> 2) * C::BLK + (ks & 3) * 32) >> 4;
           umma_bf16(tmem + C::TM_R + 128, dV_k0 + off, dO_k0 + off, id_s, ks > 0 ? 1u : 0u);
         }
@@ -229,7 +239,7 @@ __global__ void __launch_bounds__(512, 1)
             break;
           tc_fence_after();
 #pragma unroll
-          for (int ks = 0; ks < 8; ks++) {
+          for (int ks = 0; ks < KD; ks++) {
             const uint32_t off = ((ks >> 2) * C::BLK + (ks & 3) * 32) >> 4;
             umma_bf16(tmem + rB, dK_k + off, dQ_k + st1 + off, id_s, ks > 0 ? 1u : 0u);
           }
@@ -256,7 +266,7 @@ __global__ void __launch_bounds__(512, 1)
           if (!(ok = mbar_wait(&bars->r_free, i & 1, wd))) break;
           tc_fence_after();
 #pragma unroll
-          for (int ks = 0; ks < 8; ks++) {
+          for (int ks = 0; ks < KD; ks++) {
             const uint32_t off = ((ks >> 2) * C::BLK + (ks & 3) * 32) >> 4;
             umma_bf16(tmem + rA, dV_k + off, dO_k + st1 + off, id_s, ks > 0 ? 1u : 0u);
           }
@@ -374,6 +384,8 @@ __global__ void __launch_bounds__(512, 1)
       __nv_bfloat16* dst = p.dv + ((seq0 + kvc) * p.H + h) * D + qh;
 #pragma unroll 1
       for (int c = 0; c < 2; c++) {
+        const int nvalid = D - (qh + c * 32);  // columns of this chunk inside d (d = 80: 32, 32, 16, none)
+        if (nvalid <= 0) break;
         uint32_t v[32];
         tmem_ld32(tl + C::TM_DV + qh + c * 32, v);
         tmem_ld_wait(v);
@@ -381,7 +393,7 @@ __global__ void __launch_bounds__(512, 1)
           float f[32];
 #pragma unroll
           for (int e = 0; e < 32; e++) f[e] = __uint_as_float(v[e]);
-          store_row32(dst + c * 32, f);
+          store_row(dst + c * 32, f, nvalid < 32 ? nvalid : 32);
         }
       }
     }
@@ -391,7 +403,8 @@ __global__ void __launch_bounds__(512, 1)
     const int w = warp & 3;                       // column chunk d = 32 w .. 32 w + 31
     const uint32_t tl = tmem + ((uint32_t)(w * 32) << 16);
     float* stg = sSTG + w * (32 * 32);            // this warp's [32 q][32] staging slice
-    float* acc_w = p.dq_acc + (vec0 * 4 + (long long)w * p.L128) * 32;  // chunk w of this (b, h)
+    float* acc_w = p.dq_acc + (vec0 * C::NCH + (long long)w * p.L128) * 32;  // chunk w of this (b, h)
+    const bool drains = w < C::NCH;               // d = 80: the fourth chunk (rows 96..127 of dQ^T) is zero
     bool ok = true;
     for (int i = 0; i < nq; i++) {
       ok = __all_sync(0xffffffffu, mbar_wait(&bars->dq_full, i & 1, wd));
@@ -406,6 +419,7 @@ __global__ void __launch_bounds__(512, 1)
       tc_fence_before();
       mbar_arrive(&bars->r_free);
       const int q0 = (m_lo + i) * BQ;
+      if (!drains) continue;
 #pragma unroll
       for (int c = 0; c < 4; c++) {
         if (lane == 0) bulk_wait_read<0>();  // this warp's previous reduction has read its slice
@@ -429,12 +443,13 @@ __global__ void __launch_bounds__(512, 1)
       const int kvc = kv < p.L ? kv : p.L - 1;
       __nv_bfloat16* dst = p.dk + ((seq0 + kvc) * p.H + h) * D;
 #pragma unroll 1
-      for (int c = 0; c < D / 32; c++) {
+      for (int c = 0; c < C::NCH; c++) {
         uint32_t v[32];
         tmem_ld32(tl + C::TM_DK + c * 32, v);
         tmem_ld_wait(v);
         // With RoPE, R^T per pair from the warp-coalesced (cos, sin) table.
-        if (kv < p.L) store_dk_row32(dst + c * 32, v, p.scale, p.rope_tab, kv, D, c * 8);
+        if (kv < p.L)
+          store_dk_row32(dst + c * 32, v, p.scale, p.rope_tab, kv, D, c * 8, D - c * 32 < 32 ? D - c * 32 : 32);
       }
     }
   }
@@ -449,18 +464,26 @@ __global__ void __launch_bounds__(512, 1)
   }
 }
 
-cudaError_t launch_attn_bwd_main_d128(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
-                                      const CUtensorMap& tdo, const BwdParams& p, cudaStream_t stream) {
+template <int DH>
+static cudaError_t launch_big(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
+                              const CUtensorMap& tdo, const BwdParams& p, cudaStream_t stream) {
+  using C = BwdBig<DH>;
   static bool attr_set = false;
   if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(attn_bwd_main_d128_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         Bwd128::SMEM_BYTES);
+    cudaError_t e = cudaFuncSetAttribute(attn_bwd_main_d128_kernel<DH>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         C::SMEM_BYTES);
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
   dim3 grid(p.nkt, p.H, p.B);
-  attn_bwd_main_d128_kernel<<<grid, Bwd128::THREADS, Bwd128::SMEM_BYTES, stream>>>(tq, tk, tv, tdo, p);
+  attn_bwd_main_d128_kernel<DH><<<grid, C::THREADS, C::SMEM_BYTES, stream>>>(tq, tk, tv, tdo, p);
   return cudaGetLastError();
+}
+
+cudaError_t launch_attn_bwd_main_d128(int d, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
+                                      const CUtensorMap& tdo, const BwdParams& p, cudaStream_t stream) {
+  if (d == 80) return launch_big<80>(tq, tk, tv, tdo, p, stream);
+  return launch_big<128>(tq, tk, tv, tdo, p, stream);
 }
 
 }  // namespace ddattn

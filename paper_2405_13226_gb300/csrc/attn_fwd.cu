@@ -18,6 +18,10 @@
 //              so the tensor core computes S_{j+1} while the softmax warps
 //              work on S_j.
 // TMEM: S buffers at columns 0 and 128 (P over their first 64 columns), O at 256.
+// Head dims 64, 80, 128. Tiles are stored as 64-column swizzle blocks; for
+// d = 80 the second block holds columns 64..79 and TMA zero fill beyond, and
+// the contractions run at their true sizes (5 K-steps of 16 for QK^T, N = 80
+// for PV).
 #include "common.cuh"
 
 namespace ddattn {
@@ -25,7 +29,9 @@ namespace ddattn {
 template <int D>
 struct FwdCfg {
   static constexpr int BM = 128, BN = 128, STAGES = 3;
-  static constexpr int DB = D / 64;                    // 64-column swizzle blocks per row
+  static constexpr int DB = (D + 63) / 64;             // 64-column swizzle blocks per row (d = 80: the
+                                                       // second block's columns 80..127 are TMA zero fill)
+  static constexpr int DCH = (D + 31) / 32;            // 32-column TMEM chunks of O (the last may be partial)
   static constexpr int Q_BLK = BM * 128;               // bytes of one [128 rows][64] block
   static constexpr int KV_BLK = BN * 128;
   static constexpr int Q_BYTES = DB * Q_BLK;
@@ -262,7 +268,7 @@ __global__ void __launch_bounds__(224, 1)
         if (!ok) break;
         tc_fence_after();
 #pragma unroll 1
-        for (int c = 0; c < D / 32; c++) {
+        for (int c = 0; c < C::DCH; c++) {  // columns past D of the last chunk are unused TMEM
           uint32_t ov[32];
           tmem_ld32(tl + C::TMEM_O + c * 32, ov);
           tmem_ld_wait(ov);
@@ -283,14 +289,16 @@ __global__ void __launch_bounds__(224, 1)
       const float m_use = (m_run == -INFINITY) ? 0.f : m_run;
       __nv_bfloat16* orow = p.o + (((long long)b * p.L + rowc) * p.H + h) * D;
 #pragma unroll 1
-      for (int c = 0; c < D / 32; c++) {
+      for (int c = 0; c < C::DCH; c++) {
         uint32_t ov[32];
         tmem_ld32(tl + C::TMEM_O + c * 32, ov);
         tmem_ld_wait(ov);
         if (row < p.L) {
           uint4* dst = reinterpret_cast<uint4*>(orow + c * 32);
+          const int nv = (D - c * 32 >= 32) ? 4 : (D - c * 32) / 8;  // 16-byte stores in this chunk
 #pragma unroll
           for (int q = 0; q < 4; q++) {
+            if (q >= nv) break;
             uint4 w;
             w.x = pack_bf16x2(__uint_as_float(ov[8 * q + 0]) * inv_l, __uint_as_float(ov[8 * q + 1]) * inv_l);
             w.y = pack_bf16x2(__uint_as_float(ov[8 * q + 2]) * inv_l, __uint_as_float(ov[8 * q + 3]) * inv_l);
@@ -331,6 +339,7 @@ static cudaError_t launch_fwd_d(const CUtensorMap& tq, const CUtensorMap& tk, co
 cudaError_t launch_attn_fwd(int d, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
                             const FwdParams& p, cudaStream_t stream) {
   if (d == 64) return launch_fwd_d<64>(tq, tk, tv, p, stream);
+  if (d == 80) return launch_fwd_d<80>(tq, tk, tv, p, stream);
   return launch_fwd_d<128>(tq, tk, tv, p, stream);
 }
 

@@ -98,31 +98,34 @@ __device__ __forceinline__ void rope_unrotate_pair(float& g0, float& g1, float c
   g1 = b;
 }
 
-// 32 fp32 values -> 32 bf16 at dst (16-byte aligned).
-__device__ __forceinline__ void store_row32(__nv_bfloat16* dst, const float (&f)[32]) {
+// The first n (16 or 32) of 32 fp32 values -> bf16 at dst (16-byte aligned).
+__device__ __forceinline__ void store_row(__nv_bfloat16* dst, const float (&f)[32], int n) {
   uint4* d4 = reinterpret_cast<uint4*>(dst);
 #pragma unroll
-  for (int q = 0; q < 4; q++)
+  for (int q = 0; q < 4; q++) {
+    if (8 * q >= n) break;
     d4[q] = make_uint4(pack_bf16x2(f[8 * q], f[8 * q + 1]), pack_bf16x2(f[8 * q + 2], f[8 * q + 3]),
                        pack_bf16x2(f[8 * q + 4], f[8 * q + 5]), pack_bf16x2(f[8 * q + 6], f[8 * q + 7]));
+  }
 }
 
-// One 32-column slice of a dK row: dk = scale * acc, then R^T at position m
-// when tab != nullptr (pair-pairs jj0 .. jj0 + 7 of the table above).
+// One slice of a dK row (n = 16 or 32 columns): dk = scale * acc, then R^T at
+// position m when tab != nullptr (pair-pairs jj0 .. jj0 + n/4 - 1 of the table above).
 __device__ __forceinline__ void store_dk_row32(__nv_bfloat16* dst, const uint32_t (&v)[32], float sc,
-                                               const float4* tab, int m, int d, int jj0) {
+                                               const float4* tab, int m, int d, int jj0, int n) {
   float f[32];
 #pragma unroll
   for (int e = 0; e < 32; e++) f[e] = __uint_as_float(v[e]) * sc;
   if (tab) {
 #pragma unroll
     for (int u = 0; u < 8; u++) {
+      if (4 * u >= n) break;
       const float4 cs = tab[rope_tab_index(m, d, jj0 + u)];
       rope_unrotate_pair(f[4 * u], f[4 * u + 1], cs.x, cs.y);
       rope_unrotate_pair(f[4 * u + 2], f[4 * u + 3], cs.z, cs.w);
     }
   }
-  store_row32(dst, f);
+  store_row(dst, f, n);
 }
 
 struct FwdParams {
@@ -146,7 +149,7 @@ struct BwdParams {
   const float* lse;
   float* lse2_pad;  // [B, H, L128]: LSE * log2(e); +inf past L
   float* delta_pad; // [B, H, L128]: D_i = <dO_i, o_i>; 0 past L
-  float* dq_acc;    // [B, H, L128, d] fp32
+  float* dq_acc;    // fp32: [B, H, L128, 64] for d = 64, else [B, H, ceil(d/32), L128, 32]
   __nv_bfloat16* dq;
   __nv_bfloat16* dk;
   __nv_bfloat16* dv;
@@ -170,7 +173,7 @@ struct RopeParams {
 // Launchers (defined in attn_fwd.cu / attn_bwd.cu / rope.cu); return a cudaError_t.
 cudaError_t launch_attn_fwd(int d, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
                             const FwdParams& p, cudaStream_t stream);
-cudaError_t launch_attn_bwd_main_d128(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
+cudaError_t launch_attn_bwd_main_d128(int d, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
                                       const CUtensorMap& tdo, const BwdParams& p, cudaStream_t stream);
 cudaError_t launch_attn_bwd(int d, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
                             const CUtensorMap& tdo, const BwdParams& p, int phases, cudaStream_t stream);

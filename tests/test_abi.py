@@ -47,6 +47,8 @@ def test_workspace_sizes(lib):
     ragged = lib.make_desc(3, 200, 2, 128)
     assert lib.workspace_size(ragged, True) == 256 + 2 * 3 * 2 * 256 * 4 + 3 * 2 * 256 * 128 * 4
     assert lib.workspace_size(lib.make_desc(1, 128, 1, 96), True) == 0       # unsupported head dim
+    # d = 80: accumulator in 3 chunks of 32 columns
+    assert lib.workspace_size(lib.make_desc(3, 200, 2, 80), True) == 256 + 2 * 3 * 2 * 256 * 4 + 3 * 2 * 256 * 96 * 4
     assert lib.workspace_size(lib.make_desc(0, 128, 1, 64), True) == 0       # empty batch
 
 
@@ -63,7 +65,7 @@ def test_host_validation_before_launch(lib):
     assert _fwd(lib, d, good, ws=None) == lib.DD_ERR_WORKSPACE                  # no workspace
     assert _fwd(lib, d, good, ws=0x100010) == lib.DD_ERR_WORKSPACE              # workspace not 256-aligned
     assert _fwd(lib, d, good, ws_bytes=16) == lib.DD_ERR_WORKSPACE              # workspace too small
-    assert _fwd(lib, lib.make_desc(2, 256, 2, 80), good) == lib.DD_ERR_UNSUPPORTED
+    assert _fwd(lib, lib.make_desc(2, 256, 2, 96), good) == lib.DD_ERR_UNSUPPORTED
     assert _fwd(lib, lib.make_desc(2, 0, 2, 128), good) == lib.DD_ERR_INVALID_ARG
     bad_scale = lib.make_desc(2, 256, 2, 128)
     bad_scale.scale = float("nan")
@@ -99,5 +101,5 @@ def test_rope_qk_host_validation(lib):
     assert call(lib.make_desc(2, 256, 2, 128), p) == lib.DD_ERR_INVALID_ARG        # rope_base = 0
     assert call(d, [None] + p[1:]) == lib.DD_ERR_INVALID_ARG                      # null q
     assert call(d, p[:3] + [0x40004]) == lib.DD_ERR_INVALID_ARG                   # misaligned k_rot
-    assert call(lib.make_desc(2, 256, 2, 80, rope_base=1e4), p) == lib.DD_ERR_UNSUPPORTED
+    assert call(lib.make_desc(2, 256, 2, 96, rope_base=1e4), p) == lib.DD_ERR_UNSUPPORTED
     assert L.dd_rope_qk(None, *p, None) == lib.DD_ERR_INVALID_ARG
