@@ -107,6 +107,19 @@ def test_dm_baseline_full_size(seed):
         np.testing.assert_array_equal(o_bits[b, i], vb[b, i])
 
 
+def test_dm_short_chunks_full_size():
+    """Concat-and-chunk at 32 chunks x 2048 (H=16, d=128): the short-sequence
+    forward path with document offsets over thousands of query tiles."""
+    off = wl.concat_and_chunk_offsets(9, n_chunks=32, chunk=2048)
+    qb, kb, vb, gb = _inputs(32, 2048, 16, 128, seed=9)
+    gpu = run_cuda(qb, kb, vb, gb, default_scale(128), off)
+    errs = check_sampled(qb, kb, vb, gb, default_scale(128), [(0, 0), (31, 15), (17, 6)], off, n_rand=6, gpu=gpu)
+    print(errs)
+    o_bits = gpu[0].view(__import__("torch").int16).cpu().numpy().view(np.uint16)
+    for (b, i) in doc_start_rows(32, 2048, off):
+        np.testing.assert_array_equal(o_bits[b, i], vb[b, i])
+
+
 @pytest.mark.parametrize("seed", [0, 3])
 def test_pack8k_dm_full_size(seed):
     """Pack-8k+DM: best-fit-decreasing bins of 8192 tokens with masked pad tails."""
