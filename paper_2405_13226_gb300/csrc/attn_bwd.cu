@@ -78,63 +78,96 @@ template <int D>
 __host__ __device__ constexpr int acc_cols() { return D == 64 ? 64 : (D + 31) / 32 * 32; }
 
 // ------------------------------------------------------------------ pre
-// One group of G threads per (b, i, h) row, rows in memory order; the first
-// d/8 threads of a group load 8 bf16 each (G = d/8 rounded up to a power of
-// two, the shuffle width).
+// D_i = <dO_i, o_i>: one group of G threads per (b, i, h) row, rows in memory
+// order; the first d/8 threads of a group load 8 bf16 each (G = d/8 rounded up
+// to a power of two, the shuffle width). A warp covers 32/G rows per step and
+// keeps U steps of loads in flight before reducing; each step also zeroes the
+// same number of the fp32 dQ accumulator's rows (taken as a flat array), so
+// reads and writes share the memory bus (measured 0.172 ms for 1.07 GB at
+// H = 16, d = 128, 65536 tokens, vs 0.190 with the zeroing as a separate pass).
+// LSE*log2e and the padded rows then go over [B, H, L128] in memory order, and
+// the accumulator rows beyond B*L*H are zeroed.
 template <int D>
 __global__ void __launch_bounds__(256) attn_bwd_pre_kernel(const BwdParams p) {
   constexpr int NP = D / 8;                                        // 16-byte parts per row
   constexpr int G = NP <= 8 ? 8 : (NP <= 16 ? 16 : 32);            // threads per row
+  constexpr int RPW = 32 / G;                                      // rows per warp step
+  constexpr int U = 4;                                             // warp steps in flight
   const long long nrows = (long long)p.B * p.L * p.H;
-  const long long total = nrows * G;
   const long long tid = (long long)blockIdx.x * blockDim.x + threadIdx.x;
   const long long stride = (long long)gridDim.x * blockDim.x;
-  const int lane = threadIdx.x & 31;
+  const int lane = threadIdx.x & 31, sub = lane / G, part = lane % G;
+  const long long warp = tid >> 5, nwarps = stride >> 5;
   // The loop bound is uniform per warp so every shuffle sees all 32 lanes.
-  for (long long base = tid - lane; base < total; base += stride) {
-    const long long t = base + lane;
-    const bool valid = t < total;
-    const long long row = valid ? t / G : 0;
-    const int part = (int)(t % G);
-    float acc = 0.f;
-    if (valid && part < NP) {
-      const uint4 a = reinterpret_cast<const uint4*>(p.o + row * D)[part];
-      const uint4 g = reinterpret_cast<const uint4*>(p.dO + row * D)[part];
-      const __nv_bfloat162* a2 = reinterpret_cast<const __nv_bfloat162*>(&a);
-      const __nv_bfloat162* g2 = reinterpret_cast<const __nv_bfloat162*>(&g);
+  for (long long r0 = warp * (RPW * U); r0 < nrows; r0 += nwarps * (RPW * U)) {
+    uint4 a[U], g[U];
+#pragma unroll
+    for (int u = 0; u < U; u++) {
+      const long long row = r0 + u * RPW + sub;
+      if (row < nrows && part < NP) {
+        a[u] = reinterpret_cast<const uint4*>(p.o + row * D)[part];
+        g[u] = reinterpret_cast<const uint4*>(p.dO + row * D)[part];
+      } else {
+        a[u] = make_uint4(0u, 0u, 0u, 0u);
+        g[u] = make_uint4(0u, 0u, 0u, 0u);
+      }
+    }
+    {  // zero the accumulator span of these rows (flat), interleaving writes with the reads
+      constexpr int AC = acc_cols<D>();
+      float4* acc4 = reinterpret_cast<float4*>(p.dq_acc) + r0 * (AC / 4);
+      const long long lim = (nrows - r0 < RPW * U ? nrows - r0 : RPW * U) * (AC / 4);
+#pragma unroll
+      for (int k = 0; k < RPW * U * AC / 4 / 32; k++)
+        if (k * 32 + lane < lim) acc4[k * 32 + lane] = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+    float acc[U];
+#pragma unroll
+    for (int u = 0; u < U; u++) {
+      const __nv_bfloat162* a2 = reinterpret_cast<const __nv_bfloat162*>(&a[u]);
+      const __nv_bfloat162* g2 = reinterpret_cast<const __nv_bfloat162*>(&g[u]);
+      acc[u] = 0.f;
 #pragma unroll
       for (int e = 0; e < 4; e++) {
         const float2 x = __bfloat1622float2(a2[e]);
         const float2 y = __bfloat1622float2(g2[e]);
-        acc = fmaf(x.x, y.x, acc);
-        acc = fmaf(x.y, y.y, acc);
+        acc[u] = fmaf(x.x, y.x, acc[u]);
+        acc[u] = fmaf(x.y, y.y, acc[u]);
       }
     }
 #pragma unroll
-    for (int off = G / 2; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off, G);
-    if (valid && part == 0) {
-      const int h = (int)(row % p.H);
-      const long long bi = row / p.H;
-      const int i = (int)(bi % p.L);
-      const int b = (int)(bi / p.L);
-      const long long o = ((long long)b * p.H + h) * p.L128 + i;
-      p.delta_pad[o] = acc;
-      p.lse2_pad[o] = p.lse[((long long)b * p.H + h) * p.L + i] * kLog2e;
+    for (int u = 0; u < U; u++)
+#pragma unroll
+      for (int off = G / 2; off > 0; off >>= 1) acc[u] += __shfl_xor_sync(0xffffffffu, acc[u], off, G);
+    if (part == 0) {
+#pragma unroll
+      for (int u = 0; u < U; u++) {
+        const long long row = r0 + u * RPW + sub;
+        if (row < nrows) {
+          const int h = (int)(row % p.H);
+          const long long bi = row / p.H;
+          const int i = (int)(bi % p.L);
+          const int b = (int)(bi / p.L);
+          p.delta_pad[((long long)b * p.H + h) * p.L128 + i] = acc[u];
+        }
+      }
     }
   }
-  // padding rows i in [L, L128)
-  const int pad = p.L128 - p.L;
-  const long long npad = (long long)p.B * p.H * pad;
-  for (long long t = tid; t < npad; t += stride) {
-    const long long bh = t / pad;
-    const long long o = bh * p.L128 + p.L + (t % pad);
-    p.delta_pad[o] = 0.f;
-    p.lse2_pad[o] = INFINITY;
+  // LSE * log2(e) over [B, H, L128]; rows past L: LSE = +inf (P = 0), D = 0.
+  const long long nvec = (long long)p.B * p.H * p.L128;
+  for (long long t = tid; t < nvec; t += stride) {
+    const long long bh = t / p.L128;
+    const int i = (int)(t - bh * p.L128);
+    if (i < p.L) {
+      p.lse2_pad[t] = p.lse[bh * p.L + i] * kLog2e;
+    } else {
+      p.lse2_pad[t] = INFINITY;
+      p.delta_pad[t] = 0.f;
+    }
   }
-  // zero the dQ accumulator
+  // zero the rest of the dQ accumulator (past nrows * acc_cols: the padded rows)
   const long long n4 = (long long)p.B * p.H * p.L128 * acc_cols<D>() / 4;
   float4* acc4 = reinterpret_cast<float4*>(p.dq_acc);
-  for (long long t = tid; t < n4; t += stride) acc4[t] = make_float4(0.f, 0.f, 0.f, 0.f);
+  for (long long t = nrows * (acc_cols<D>() / 4) + tid; t < n4; t += stride) acc4[t] = make_float4(0.f, 0.f, 0.f, 0.f);
 }
 
 // ------------------------------------------------------------------ post
