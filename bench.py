@@ -73,16 +73,23 @@ def load_peaks():
 
 
 # ------------------------------------------------------------------ dist
-def dist_setup(n_gpus):
+def dist_setup(n_gpus, backend=None):
+    """Rank, world size and local rank from the torchrun environment; for N > 1
+    one process group over NCCL (one GPU per rank), or `backend` if given
+    (the CPU tests use gloo)."""
     import torch
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
+    backend = backend or "nccl"
     if world > 1:
         import torch.distributed as dist
-        torch.cuda.set_device(local)
-        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
-    else:
+        if backend == "nccl":
+            torch.cuda.set_device(local)
+            dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+        else:
+            dist.init_process_group(backend)
+    elif backend == "nccl":
         torch.cuda.set_device(0)
     return rank, world, local
 
@@ -94,13 +101,21 @@ def barrier(world):
 
 
 def max_over_ranks(x, world):
+    """The slowest rank's time: every rank's CUDA-event time, reduced with MAX."""
     if world == 1:
         return x
     import torch
     import torch.distributed as dist
-    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
     return float(t.item())
+
+
+def replica_value(flops_per_step, steps, total_ms, world):
+    """Whole-job TFLOP/s of N replicas: every rank runs the same per-rank
+    workload (weak scaling), timed by the slowest rank."""
+    return world * flops_per_step * steps / (total_ms * 1e-3) / 1e12
 
 
 # ------------------------------------------------------------------ clocks
@@ -300,7 +315,7 @@ def run_ours(args):
 
     step_flops = sum(bk.flops for bk in buckets)
     ms_per_step = total_ms / args.steps
-    value = world * step_flops * args.steps / (total_ms * 1e-3) / 1e12
+    value = replica_value(step_flops, args.steps, total_ms, world)
 
     per_bucket, fwd_t, main_t, main_flops = [], 0.0, 0.0, 0
     for i, bk in enumerate(buckets):
@@ -560,6 +575,23 @@ def e2e_measure(ddattn, qb, kb, vb, gb, buckets, stream, dev, args, world):
     steps = max(2, min(args.steps, 5))
     run(2 * len(buckets))
     torch.cuda.synchronize()
+    # the host link alone: one call's input and output copies, concurrently
+    call0 = sets[0][1][-1]
+    e0, e1, e2 = (torch.cuda.Event(enable_timing=True) for _ in range(3))
+    e0.record(s_in)
+    s_out.wait_event(e0)
+    with torch.cuda.stream(s_in):
+        for hsrc, d in zip(host_in, sets[0][0]):
+            d.copy_(hsrc, non_blocking=True)
+    with torch.cuda.stream(s_out):
+        for n in outs:
+            host_out[n].copy_(getattr(call0, n).view(T, H, D), non_blocking=True)
+        host_lse.copy_(call0.lse.view(-1), non_blocking=True)
+    e1.record(s_in)
+    e2.record(s_out)
+    torch.cuda.synchronize()
+    link_ms = max(e0.elapsed_time(e1), e0.elapsed_time(e2))
+    call_bytes = 4 * T * H * D * 2 + (4 * T * H * D * 2 + T * H * 4)
     barrier(world)
     s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     s.record(s_in)
@@ -571,8 +603,11 @@ def e2e_measure(ddattn, qb, kb, vb, gb, buckets, stream, dev, args, world):
     flops = sum(bk.flops for bk in buckets)
     h2d = len(buckets) * 4 * T * H * D * 2
     d2h = len(buckets) * (4 * T * H * D * 2 + T * H * 4)
+    link_gbps = call_bytes / (link_ms * 1e-3) / 1e9
     return {"value": world * flops / (ms * 1e-3) / 1e12, "unit": "TFLOP/s", "ms_per_step": ms,
             "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+            "host_link_GBps_in_plus_out": link_gbps,
+            "copy_bound_ms_per_step": (h2d + d2h) / (link_gbps * 1e9) * 1e3,
             "how": "per bucket call: pinned host q,k,v,dO -> device, fwd+bwd via the C ABI, o,lse,dq,dk,dv -> "
                    "pinned host; copies in / kernels / copies out on 3 streams, 2 device buffer sets"}
 
