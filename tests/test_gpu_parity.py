@@ -138,3 +138,34 @@ def test_long_context_full_size():
     qb, kb, vb, gb = _inputs(4, 16384, 32, 128, qk_mult=3.0)
     errs = check_sampled(qb, kb, vb, gb, default_scale(128), [(0, 0), (3, 31)], n_rand=4)
     print(errs)
+
+
+def test_every_token_its_own_document():
+    """Degenerate document mask: each token is a one-token document, so every row
+    attends only to itself: o = v and dv = dO exactly (P = 1), and dq, dk vanish up
+    to the rounding of dS = P (dP - D), whose two fp32 dot products of the same
+    vectors are summed in different orders."""
+    import torch
+    B, L, H, d = 2, 300, 2, 128
+    off = np.arange(0, B * L + 1, dtype=np.int32)
+    qb, kb, vb, gb = _inputs(B, L, H, d, seed=12)
+    o, lse, dq, dk, dv = run_cuda(qb, kb, vb, gb, default_scale(d), off)
+    np.testing.assert_array_equal(o.view(torch.int16).cpu().numpy().view(np.uint16), vb)
+    assert float(dq.float().abs().max()) < 1e-4 and float(dk.float().abs().max()) < 1e-4
+    np.testing.assert_array_equal(dv.view(torch.int16).cpu().numpy().view(np.uint16), gb)
+
+
+def test_longest_document_full_size():
+    """One 65536-token sequence (the longest document of the length model), H=1:
+    the largest positions and tile counts; sampled rows against the oracle."""
+    qb, kb, vb, gb = _inputs(1, 65536, 1, 128, seed=13)
+    errs = check_sampled(qb, kb, vb, gb, default_scale(128), [(0, 0)], n_rand=6)
+    print(errs)
+
+
+def test_many_short_sequences():
+    """B = 32768 sequences of L = 8 (H = 2, d = 64): a grid of 32768 x 2 CTAs of
+    one ragged tile each."""
+    qb, kb, vb, gb = _inputs(32768, 8, 2, 64, seed=14)
+    errs = check_sampled(qb, kb, vb, gb, default_scale(64), [(0, 0), (32767, 1), (12345, 0)], n_rand=2)
+    print(errs)
