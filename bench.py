@@ -367,7 +367,8 @@ def run_ours(args):
         "roofline": roofline,
         "cpu_baseline": cpu,
         "e2e": e2e,
-        "gpu_launches": args.steps * nb * 4,
+        # per bucket call: forward, backward pre / main / post (+ RoPE rotation and table)
+        "gpu_launches": args.steps * nb * (4 + (2 if args.rope_base else 0)),
         "clocks": clk.summary(),
     }
     line.update(extras)
