@@ -6,9 +6,8 @@
 //   S^T  = K Q_i^T            P^T  = exp2(S^T * scale * log2e - LSE_i * log2e)  (masked)
 //   dP^T = V dO_i^T           dS^T = P^T (dP^T - D_i)
 //   dV  += P^T dO_i           dK  += dS^T Q_i           dQ_i^T = K^T dS^T
-// All five contractions are M = 128, N = 128 UMMAs issued by one thread: an
-// instruction costs about the same for any N <= 256, so 128-row query steps
-// give each instruction twice the work of 64-row steps.
+// All five contractions are M = 128, N = 128 UMMAs issued by one thread
+// (128-row query steps: an N = 64 instruction costs ~80% of an N = 128 one).
 //
 // TMEM (512 columns): two 128-column regions R[0], R[1] whose roles alternate
 // every step (A = R[i % 2], B = R[(i + 1) % 2]):
