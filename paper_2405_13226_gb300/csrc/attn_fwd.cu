@@ -13,11 +13,14 @@
 //              in bf16/fp32).
 //   warp 4     TMA producer for Q (once) and K tiles (3-stage ring); TMEM alloc.
 //   warp 5     TMA producer for V tiles (3-stage ring).
-//   warp 6     one thread issues tcgen05.mma: S[j%2] = Q K_j^T (TMEM, fp32),
+//   warp 6     one thread issues tcgen05.mma: S[j%3] = Q K_j^T (TMEM, fp32),
 //              then O += P_{j-1} V_{j-1} with P read from TMEM (the .ts form),
 //              so the tensor core computes S_{j+1} while the softmax warps
 //              work on S_j.
-// TMEM: S buffers at columns 0 and 128 (P over their first 64 columns), O at 256.
+// TMEM: three S buffers at columns 0, 128, 256 (P over their first 64 columns),
+// O at 384. With three, S_{j+2} goes to a buffer whose PV finished a tile ago,
+// so the MMA thread never waits for the PV it has just issued (with two it
+// did, leaving the tensor pipe idle for a PV's duration every tile).
 // Head dims 64, 80, 128. Tiles are stored as 64-column swizzle blocks; for
 // d = 80 the second block holds columns 64..79 and TMA zero fill beyond, and
 // the contractions run at their true sizes (5 K-steps of 16 for QK^T, N = 80
@@ -41,8 +44,11 @@ struct FwdCfg {
   static constexpr int OFF_V = OFF_K + STAGES * KV_BYTES;
   static constexpr int OFF_BAR = OFF_V + STAGES * KV_BYTES;
   static constexpr int SMEM_BYTES = OFF_BAR + 256 + 1024;
-  static constexpr uint32_t TMEM_S = 0;                // S buffers at columns 0 and 128
-  static constexpr uint32_t TMEM_O = 256;              // O: D columns
+  static constexpr int PF = 4;                         // K / V tiles prefetched into L2 ahead of the ring
+  static constexpr int NS = 3;                         // S buffers (P of tile j lives in buffer j % 3
+                                                       // until PV_j has read it)
+  static constexpr uint32_t TMEM_S = 0;                // S buffers at columns 0, 128, 256
+  static constexpr uint32_t TMEM_O = 384;              // O: D columns
   static constexpr uint32_t TMEM_COLS = 512;
   static constexpr int THREADS = 224;
 };
@@ -50,7 +56,7 @@ struct FwdCfg {
 struct FwdBars {
   uint64_t q_full;
   uint64_t k_full[3], k_empty[3], v_full[3], v_empty[3];
-  uint64_t s_full[2], p_full[2], pv_done[2];
+  uint64_t s_full[3], p_full[3], pv_done[3];
   uint64_t mma_drain;
   uint32_t tmem_base;
   int abort_flag;
@@ -88,7 +94,7 @@ __global__ void __launch_bounds__(224, 1)
       mbar_init(&bars->v_full[i], 1);
       mbar_init(&bars->v_empty[i], 1);
     }
-    for (int i = 0; i < 2; i++) {
+    for (int i = 0; i < C::NS; i++) {
       mbar_init(&bars->s_full[i], 1);
       mbar_init(&bars->p_full[i], 128);
       mbar_init(&bars->pv_done[i], 1);
@@ -123,6 +129,8 @@ __global__ void __launch_bounds__(224, 1)
         const int kv0 = (n_lo + j) * C::BN;
         for (int blk = 0; blk < C::DB; blk++)
           tma_load_4d(sK + s * C::KV_BYTES + blk * C::KV_BLK, &tmK, &bars->k_full[s], 64 * blk, h, kv0, b);
+        if (j + C::PF < nt)  // K tile j + PF into L2: the ring alone does not cover the load latency
+          for (int blk = 0; blk < C::DB; blk++) tma_prefetch_4d(&tmK, 64 * blk, h, kv0 + C::PF * C::BN, b);
         issued = j + 1;
       }
       if (*wd.abort_flag) {  // let in-flight copies land before the CTA exits
@@ -143,6 +151,8 @@ __global__ void __launch_bounds__(224, 1)
         const int kv0 = (n_lo + j) * C::BN;
         for (int blk = 0; blk < C::DB; blk++)
           tma_load_4d(sV + s * C::KV_BYTES + blk * C::KV_BLK, &tmV, &bars->v_full[s], 64 * blk, h, kv0, b);
+        if (j + C::PF < nt)
+          for (int blk = 0; blk < C::DB; blk++) tma_prefetch_4d(&tmV, 64 * blk, h, kv0 + C::PF * C::BN, b);
         issued = j + 1;
       }
       if (*wd.abort_flag)
@@ -154,36 +164,42 @@ __global__ void __launch_bounds__(224, 1)
     if (lane == 0) {
       constexpr uint32_t idesc_s = idesc_bf16(128, 128, false, false);  // Q, K both K-major
       constexpr uint32_t idesc_o = idesc_bf16(128, D, false, true);      // P (TMEM) x V (MN-major)
-      const uint32_t aQ = smem_u32(sQ), aK = smem_u32(sK), aV = smem_u32(sV);
+      // Descriptors are built once; a K-slice or ring stage is an added (byte offset >> 4)
+      // on the 14-bit start-address field (smem offsets stay below 256 KB), so each
+      // UMMA costs this thread one add instead of a descriptor rebuild.
+      const uint64_t dQ0 = sdesc_sw128(smem_u32(sQ), 16, 1024);
+      const uint64_t dK0 = sdesc_sw128(smem_u32(sK), 16, 1024);
+      const uint64_t dV0 = sdesc_sw128(smem_u32(sV), C::KV_BLK, 1024);
       if (mbar_wait(&bars->q_full, 0, wd)) {
         for (int j = 0; j <= nt; j++) {
           if (j < nt) {
-            const int ks = j % ST, sb = j & 1;
+            const int ks = j % ST, sb = j % C::NS;
             if (!mbar_wait(&bars->k_full[ks], (j / ST) & 1, wd)) break;
             // S[sb] holds P_{j-2} until PV_{j-2} has read it.
-            if (j >= 2 && !mbar_wait(&bars->pv_done[sb], ((j >> 1) - 1) & 1, wd)) break;
+            if (j >= C::NS && !mbar_wait(&bars->pv_done[sb], ((j / C::NS) - 1) & 1, wd)) break;
             tc_fence_after();
+            const uint64_t dK = dK0 + ((uint32_t)(ks * C::KV_BYTES) >> 4);
+            const uint32_t tS = tmem + C::TMEM_S + sb * 128;
 #pragma unroll
             for (int kk = 0; kk < D / 16; kk++) {
-              const uint64_t da = sdesc_sw128(aQ + (kk >> 2) * C::Q_BLK + (kk & 3) * 32, 16, 1024);
-              const uint64_t db =
-                  sdesc_sw128(aK + ks * C::KV_BYTES + (kk >> 2) * C::KV_BLK + (kk & 3) * 32, 16, 1024);
-              umma_bf16(tmem + C::TMEM_S + sb * 128, da, db, idesc_s, kk > 0 ? 1u : 0u);
+              constexpr int q_blk = C::Q_BLK, kv_blk = C::KV_BLK;
+              umma_bf16(tS, dQ0 + (uint32_t)(((kk >> 2) * q_blk + (kk & 3) * 32) >> 4),
+                        dK + (uint32_t)(((kk >> 2) * kv_blk + (kk & 3) * 32) >> 4), idesc_s, kk > 0 ? 1u : 0u);
             }
             umma_commit(&bars->s_full[sb]);
             umma_commit(&bars->k_empty[ks]);
           }
           if (j >= 1) {
-            const int i = j - 1, vs = i % ST, pb = i & 1;
+            const int i = j - 1, vs = i % ST, pb = i % C::NS;
             if (!mbar_wait(&bars->v_full[vs], (i / ST) & 1, wd)) break;
-            if (!mbar_wait(&bars->p_full[pb], (i >> 1) & 1, wd)) break;
+            if (!mbar_wait(&bars->p_full[pb], (i / C::NS) & 1, wd)) break;
             tc_fence_after();
+            const uint64_t dV = dV0 + ((uint32_t)(vs * C::KV_BYTES) >> 4);
+            const uint32_t tP = tmem + C::TMEM_S + pb * 128;
 #pragma unroll
-            for (int kk = 0; kk < C::BN / 16; kk++) {
-              const uint64_t db = sdesc_sw128(aV + vs * C::KV_BYTES + kk * 2048, C::KV_BLK, 1024);
-              umma_bf16_ts(tmem + C::TMEM_O, tmem + C::TMEM_S + pb * 128 + kk * 8, db, idesc_o,
+            for (int kk = 0; kk < C::BN / 16; kk++)
+              umma_bf16_ts(tmem + C::TMEM_O, tP + kk * 8, dV + (uint32_t)((kk * 2048) >> 4), idesc_o,
                            (i > 0 || kk > 0) ? 1u : 0u);
-            }
             umma_commit(&bars->pv_done[pb]);
             umma_commit(&bars->v_empty[vs]);
           }
@@ -204,10 +220,10 @@ __global__ void __launch_bounds__(224, 1)
     float m_run = -INFINITY, l_run = 0.f;
     bool ok = true;
     for (int j = 0; j < nt && ok; j++) {
-      const int sb = j & 1;
+      const int sb = j % C::NS;
       const int kv0 = (n_lo + j) * C::BN;
       const uint32_t sbuf = tl + C::TMEM_S + sb * 128;
-      ok = __all_sync(0xffffffffu, mbar_wait(&bars->s_full[sb], (j >> 1) & 1, wd));
+      ok = __all_sync(0xffffffffu, mbar_wait(&bars->s_full[sb], (j / C::NS) & 1, wd));
       if (!ok) break;
       tc_fence_after();
       uint32_t v0[32], v1[32], v2[32], v3[32];
@@ -264,7 +280,7 @@ __global__ void __launch_bounds__(224, 1)
       tmem_st32(sbuf + 32, pk1);
       // O *= alpha, after PV_{j-1} landed and before PV_j is issued.
       if (__any_sync(0xffffffffu, rescale)) {
-        ok = __all_sync(0xffffffffu, mbar_wait(&bars->pv_done[(j - 1) & 1], ((j - 1) >> 1) & 1, wd));
+        ok = __all_sync(0xffffffffu, mbar_wait(&bars->pv_done[(j - 1) % C::NS], ((j - 1) / C::NS) & 1, wd));
         if (!ok) break;
         tc_fence_after();
 #pragma unroll 1
@@ -282,7 +298,7 @@ __global__ void __launch_bounds__(224, 1)
       mbar_arrive(&bars->p_full[sb]);
     }
     // Epilogue: O / l -> bf16, LSE = (m + log2 l) * ln2.
-    if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&bars->pv_done[(nt - 1) & 1], ((nt - 1) >> 1) & 1, wd));
+    if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&bars->pv_done[(nt - 1) % C::NS], ((nt - 1) / C::NS) & 1, wd));
     if (ok) {
       tc_fence_after();
       const float inv_l = l_run > 0.f ? 1.f / l_run : 0.f;
