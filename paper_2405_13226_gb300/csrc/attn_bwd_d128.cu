@@ -79,15 +79,6 @@ struct Bwd128Bars {
 };
 static_assert(sizeof(Bwd128Bars) <= 256, "barrier block");
 
-template <uint32_t N>
-__device__ __forceinline__ void setmaxnreg_inc() {
-  asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(N));
-}
-template <uint32_t N>
-__device__ __forceinline__ void setmaxnreg_dec() {
-  asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(N));
-}
-
 template <int DH>
 __global__ void __launch_bounds__(512, 1)
     attn_bwd_main_d128_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,

@@ -173,8 +173,6 @@ struct RopeParams {
 // Launchers (defined in attn_fwd.cu / attn_bwd.cu / rope.cu); return a cudaError_t.
 cudaError_t launch_attn_fwd(int d, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
                             const FwdParams& p, cudaStream_t stream);
-cudaError_t launch_attn_fwd_persist(int d, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
-                                    const FwdParams& p, cudaStream_t stream);
 cudaError_t launch_attn_bwd_main_d128(int d, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
                                       const CUtensorMap& tdo, const BwdParams& p, cudaStream_t stream);
 cudaError_t launch_attn_bwd(int d, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,

@@ -159,6 +159,17 @@ __device__ __forceinline__ void bulk_reduce_add_f32(float* gdst, const void* ssr
                : "memory");
 }
 
+// Warpgroup register reallocation: every warp of the warpgroup executes it;
+// the increases must fit in what the decreases and the launch leave free.
+template <uint32_t N>
+__device__ __forceinline__ void setmaxnreg_inc() {
+  asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(N));
+}
+template <uint32_t N>
+__device__ __forceinline__ void setmaxnreg_dec() {
+  asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(N));
+}
+
 // Barrier among `count` threads (a multiple of 32) on hardware barrier `id`.
 __device__ __forceinline__ void named_bar_sync(int id, int count) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");

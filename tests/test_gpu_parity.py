@@ -34,6 +34,22 @@ def test_causal_ragged_and_edges(B, L, H, d):
     print(errs)
 
 
+@pytest.mark.parametrize("B,L,H,d", [(1, 2176, 2, 128), (1, 2300, 2, 64), (1, 2432, 1, 80)])
+def test_two_tile_forward_odd_and_ragged(B, L, H, d):
+    """More than 16 query tiles: the forward pairs consecutive query tiles in one
+    CTA. 17 tiles (the last pair has one tile), a ragged 18th tile, d = 80."""
+    errs, _ = check_full(*_inputs(B, L, H, d, seed=L), default_scale(d))
+    print(errs)
+
+
+def test_two_tile_forward_documents_on_pair_boundaries():
+    """Documents starting at the first tile of a pair (256), at the second tile of a
+    pair (384, 1152) and inside a tile, L = 2304 (18 query tiles)."""
+    off = np.array([0, 256, 384, 1000, 1152, 2304, 2304 + 129, 2 * 2304], dtype=np.int32)
+    errs, _ = check_full(*_inputs(2, 2304, 1, 128, seed=11), default_scale(128), off)
+    print(errs)
+
+
 @pytest.mark.parametrize("d", [64, 128])
 @pytest.mark.parametrize("seed", [0, 5])
 def test_document_mask_small(d, seed):
