@@ -31,9 +31,14 @@
 //             the running max grows by more than 8: P <= 256 stays exact enough
 //             in bf16 / fp32), P as bf16 pairs over the S buffer.
 //   WG2       warp 8: TMA producer for Q (both tiles, once) and the K ring, TMEM
-//             owner; warp 9: V ring producer; warp 10: one thread issues
-//             tcgen05.mma; warp 11 idle. WG2 gives registers back
-//             (setmaxnreg.dec) to the softmax groups (setmaxnreg.inc).
+//             owner; warp 9: V ring producer; warp 10: the MMA issuer; warp 11
+//             idle. WG2 gives registers back (setmaxnreg.dec) to the softmax
+//             groups (setmaxnreg.inc).
+// MMA issue: the whole of warp 10 runs the issue loop (waits, descriptor
+// arithmetic) and one lane chosen by elect.sync issues each group of MMAs and
+// its commit. The same loop run by lane 0 alone inside a divergent branch issued
+// 17% slower at L = 8192: that warp shares its SM sub-partition with two busy
+// softmax warps, and the divergent form costs more instructions per MMA.
 // TMEM (512 columns): S_t at columns 128 t, O_t at 256 + 128 t.
 // Key tiles: tile t covers [lo_t, 2u + t] (lo_t: the key tile of the document
 // start of its first row); the CTA walks the union [lo_0, 2u + 1] and each
@@ -182,8 +187,9 @@ __global__ void __launch_bounds__(384, 1)
         mbar_wait_drain(&bars->v_full[j % VST], (j / VST) & 1, wd.limit_ns);
     }
   } else if (warp == 10) {
-    // ---------------- MMA issuer
-    if (lane == 0) {
+    // ---------------- MMA issuer: the whole warp runs the loop, one elected lane issues
+    {
+      const bool leader = elect_one();
       constexpr uint32_t idesc_s = idesc_bf16(128, 128, false, false);  // Q, K both K-major
       constexpr uint32_t idesc_o = idesc_bf16(128, D, false, true);      // P (TMEM) x V (MN-major)
       // Descriptors built once; a K-slice, ring stage or tile is an added (byte offset >> 4).
@@ -201,24 +207,29 @@ __global__ void __launch_bounds__(384, 1)
           // O_t += P_t V_{j-1}
           if (ok && tile && j >= 1 && kt - 1 >= lo_t && kt - 1 <= hi_t) {
             const int i = j - 1, vs = i % VST;
-            ok = mbar_wait(&bars->v_full[vs], (i / VST) & 1, wd) && mbar_wait(&bars->p_full[t], npv[t] & 1, wd);
+            ok = __all_sync(0xffffffffu, mbar_wait(&bars->v_full[vs], (i / VST) & 1, wd) &&
+                                             mbar_wait(&bars->p_full[t], npv[t] & 1, wd));
           }
           if (ok && tile && j >= 1 && kt - 1 >= lo_t && kt - 1 <= hi_t) {
             const int i = j - 1, vs = i % VST;
             tc_fence_after();
             const uint64_t dV = dV0 + ((uint32_t)(vs * C::KV_BYTES) >> 4);
             const uint32_t tP = tmem + C::TMEM_S + t * 128;
+            if (leader) {
 #pragma unroll
-            for (int kk = 0; kk < C::BN / 16; kk++)
-              umma_bf16_ts(tmem + C::TMEM_O + t * 128, tP + kk * 8, dV + (uint32_t)((kk * 2048) >> 4), idesc_o,
-                           (npv[t] > 0 || kk > 0) ? 1u : 0u);
-            if (kt - 1 == hi_t) umma_commit(&bars->pv_done[t]);  // the tile's last PV: for the epilogue
+              for (int kk = 0; kk < C::BN / 16; kk++)
+                umma_bf16_ts(tmem + C::TMEM_O + t * 128, tP + kk * 8, dV + (uint32_t)((kk * 2048) >> 4), idesc_o,
+                             (npv[t] > 0 || kk > 0) ? 1u : 0u);
+              if (kt - 1 == hi_t) umma_commit(&bars->pv_done[t]);  // the tile's last PV: for the epilogue
+            }
+            __syncwarp();
             npv[t]++;
           }
           // S_t = Q_t K_j^T into the buffer PV_t has just read (issue order keeps them apart)
           if (ok && tile && j < NJ && kt >= lo_t && kt <= hi_t) {
             const int ks = j % KST;
-            ok = mbar_wait(&bars->k_full[ks], (j / KST) & 1, wd) && (ns[t] > 0 || mbar_wait(&bars->q_full[t], 0, wd));
+            ok = __all_sync(0xffffffffu, mbar_wait(&bars->k_full[ks], (j / KST) & 1, wd) &&
+                                             (ns[t] > 0 || mbar_wait(&bars->q_full[t], 0, wd)));
           }
           if (ok && tile && j < NJ && kt >= lo_t && kt <= hi_t) {
             const int ks = j % KST;
@@ -226,18 +237,22 @@ __global__ void __launch_bounds__(384, 1)
             const uint64_t dQ = dQ0 + ((uint32_t)(t * C::Q_BYTES) >> 4);
             const uint64_t dK = dK0 + ((uint32_t)(ks * C::KV_BYTES) >> 4);
             const uint32_t tS = tmem + C::TMEM_S + t * 128;
+            if (leader) {
 #pragma unroll
-            for (int kk = 0; kk < D / 16; kk++) {
-              constexpr int q_blk = C::Q_BLK, kv_blk = C::KV_BLK;
-              umma_bf16(tS, dQ + (uint32_t)(((kk >> 2) * q_blk + (kk & 3) * 32) >> 4),
-                        dK + (uint32_t)(((kk >> 2) * kv_blk + (kk & 3) * 32) >> 4), idesc_s, kk > 0 ? 1u : 0u);
+              for (int kk = 0; kk < D / 16; kk++) {
+                constexpr int q_blk = C::Q_BLK, kv_blk = C::KV_BLK;
+                umma_bf16(tS, dQ + (uint32_t)(((kk >> 2) * q_blk + (kk & 3) * 32) >> 4),
+                          dK + (uint32_t)(((kk >> 2) * kv_blk + (kk & 3) * 32) >> 4), idesc_s, kk > 0 ? 1u : 0u);
+              }
+              umma_commit(&bars->s_full[t]);
             }
-            umma_commit(&bars->s_full[t]);
+            __syncwarp();
             ns[t]++;
           }
         }
       }
-      umma_commit(&bars->mma_drain);
+      if (leader) umma_commit(&bars->mma_drain);
+      __syncwarp();
       mbar_wait_drain(&bars->mma_drain, 0, wd.limit_ns);
     }
   }
