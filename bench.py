@@ -41,7 +41,7 @@ PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 def kernel_source_sha1() -> str:
     import hashlib
     h = hashlib.sha1()
-    for f in ("attn_bwd_d128.cu", "common.cuh", "ptx.cuh"):
+    for f in ("attn_bwd_d128.cu", "attn_bwd_d128_persist.cu", "bwd_d128.cuh", "common.cuh", "ptx.cuh"):
         with open(os.path.join(ROOT, "paper_2405_13226_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()
@@ -54,7 +54,7 @@ def measured_traffic():
     if not os.path.exists(p):
         return None
     txt = open(p).read()
-    if "source_sha1 (attn_bwd_d128.cu + common.cuh + ptx.cuh): " + kernel_source_sha1() not in txt:
+    if "source_sha1 (attn_bwd_d128.cu + attn_bwd_d128_persist.cu + bwd_d128.cuh + common.cuh + ptx.cuh): " + kernel_source_sha1() not in txt:
         return None
     vals = []
     for line in txt.splitlines():

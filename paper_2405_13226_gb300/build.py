@@ -17,7 +17,7 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libddattn.so")
-SOURCES = ["api.cu", "attn_fwd.cu", "attn_bwd.cu", "attn_bwd_d128.cu", "rope.cu", "noalloc.cu"]
+SOURCES = ["api.cu", "attn_fwd.cu", "attn_bwd.cu", "attn_bwd_d128.cu", "attn_bwd_d128_persist.cu", "rope.cu", "noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -49,41 +49,9 @@
 // contractions over d (S^T, dP^T) take 5 K-steps instead of 8, dV and dK are
 // N = 80 UMMAs, and dQ^T stays M = 128 (its rows 80..127 are zero: K's padded
 // columns), drained by the first three warps into a 3-chunk accumulator.
-#include "common.cuh"
+#include "bwd_d128.cuh"
 
 namespace ddattn {
-
-template <int D_>
-struct BwdBig {
-  static constexpr int D = D_, BN = 128, BQ = 128;
-  static constexpr int NCH = (D + 31) / 32;              // 32-column chunks of dQ^T / dK / dV
-  static constexpr int BLK = 128 * 128;                  // [128 rows][64] bf16, 128B swizzle
-  static constexpr int TILE = 2 * BLK;                   // [128 rows][128] bf16
-  static constexpr int OFF_K = 0;
-  static constexpr int OFF_V = OFF_K + TILE;
-  static constexpr int OFF_Q = OFF_V + TILE;             // 2 stages
-  static constexpr int OFF_DO = OFF_Q + 2 * TILE;        // 2 stages (dO, then dS^T)
-  static constexpr int OFF_STG = OFF_DO + 2 * TILE;      // dQ staging quarter
-  static constexpr int STG_BYTES = 4 * 32 * 32 * 4;     // one [32 x 32] fp32 slice per drain warp
-  static constexpr int OFF_LSE = OFF_STG + STG_BYTES;    // [2][128] fp32
-  static constexpr int OFF_DEL = OFF_LSE + 2 * BQ * 4;   // [2][128] fp32
-  static constexpr int OFF_BAR = OFF_DEL + 2 * BQ * 4;
-  static constexpr int SMEM_BYTES = OFF_BAR + 256 + 1024;
-  static constexpr uint32_t TM_R = 0, TM_DV = 256, TM_DK = 384;  // R[k] at TM_R + 128 k
-  static constexpr int THREADS = 512;
-  static constexpr int REGS_LOW = 32, REGS_HIGH = 160;   // setmaxnreg split, see above
-};
-static_assert(4 * 32 * BwdBig<128>::REGS_LOW + 12 * 32 * BwdBig<128>::REGS_HIGH == 512 * 128, "register split");
-
-struct Bwd128Bars {
-  uint64_t kv_full;
-  uint64_t q_full[2], q_empty[2];
-  uint64_t s_full, dp_full, p_full, dp_read, dss_full, dv_done, dq_full, r_free;
-  uint64_t mma_done;
-  uint32_t tmem_base;
-  int abort_flag;
-};
-static_assert(sizeof(Bwd128Bars) <= 256, "barrier block");
 
 template <int DH>
 __global__ void __launch_bounds__(512, 1)
@@ -509,6 +477,10 @@ static cudaError_t launch_big(const CUtensorMap& tq, const CUtensorMap& tk, cons
 
 cudaError_t launch_attn_bwd_main_d128(int d, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
                                       const CUtensorMap& tdo, const BwdParams& p, cudaStream_t stream) {
+  // Up to 16 key tiles per sequence (L <= 2048) CTAs walk key tiles (their epilogues and
+  // the next tile's loads overlap): -26% at L = 256 ... -2.5% at L = 2048 against one CTA
+  // per key tile, which stays faster for longer sequences (+1-4% at 4096 / 8192).
+  if (p.nkt <= 16) return launch_attn_bwd_main_d128_persist(d, tq, tk, tv, tdo, p, stream);
   if (d == 80) return launch_big<80>(tq, tk, tv, tdo, p, stream);
   return launch_big<128>(tq, tk, tv, tdo, p, stream);
 }

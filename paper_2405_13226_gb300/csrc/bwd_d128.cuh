@@ -1,0 +1,71 @@
+// Shared pieces of the d = 128 / 80 backward main kernels (csrc/attn_bwd_d128.cu, one CTA
+// per key tile; csrc/attn_bwd_d128_persist.cu, CTAs walking key tiles): shared-memory and
+// TMEM layout, barrier block, work items.
+#pragma once
+#include "common.cuh"
+
+namespace ddattn {
+
+template <int D_>
+struct BwdBig {
+  static constexpr int D = D_, BN = 128, BQ = 128;
+  static constexpr int NCH = (D + 31) / 32;              // 32-column chunks of dQ^T / dK / dV
+  static constexpr int BLK = 128 * 128;                  // [128 rows][64] bf16, 128B swizzle
+  static constexpr int TILE = 2 * BLK;                   // [128 rows][128] bf16
+  static constexpr int OFF_K = 0;
+  static constexpr int OFF_V = OFF_K + TILE;
+  static constexpr int OFF_Q = OFF_V + TILE;             // 2 stages
+  static constexpr int OFF_DO = OFF_Q + 2 * TILE;        // 2 stages (dO, then dS^T)
+  static constexpr int OFF_STG = OFF_DO + 2 * TILE;      // dQ staging quarter
+  static constexpr int STG_BYTES = 4 * 32 * 32 * 4;     // one [32 x 32] fp32 slice per drain warp
+  static constexpr int OFF_LSE = OFF_STG + STG_BYTES;    // [2][128] fp32
+  static constexpr int OFF_DEL = OFF_LSE + 2 * BQ * 4;   // [2][128] fp32
+  static constexpr int OFF_BAR = OFF_DEL + 2 * BQ * 4;
+  static constexpr int SMEM_BYTES = OFF_BAR + 256 + 1024;
+  static constexpr uint32_t TM_R = 0, TM_DV = 256, TM_DK = 384;  // R[k] at TM_R + 128 k
+  static constexpr int THREADS = 512;
+  // setmaxnreg splits (4 warps low, 12 high): the per-tile kernel's, and the persistent
+  // kernel's, whose per-item state needs more registers in the producer / MMA group.
+  static constexpr int REGS_LOW = 32, REGS_HIGH = 160;
+  static constexpr int REGS_LOW_P = 48, REGS_HIGH_P = 152;
+};
+static_assert(4 * 32 * BwdBig<128>::REGS_LOW + 12 * 32 * BwdBig<128>::REGS_HIGH <= 512 * 128, "register split");
+static_assert(4 * 32 * BwdBig<128>::REGS_LOW_P + 12 * 32 * BwdBig<128>::REGS_HIGH_P <= 512 * 128, "register split");
+
+struct Bwd128Bars {
+  uint64_t kv_full;
+  uint64_t q_full[2], q_empty[2];
+  uint64_t s_full, dp_full, p_full, dp_read, dss_full, dv_done, dq_full, r_free;
+  uint64_t mma_done;
+  // the persistent kernel's item hand-offs
+  uint64_t kv_empty;          // the item's MMAs are done: K / V may be replaced
+  uint64_t dv_free, dk_free;  // the item's dV / dK have left TMEM: the next item may accumulate
+  uint64_t mma_drain;
+  uint32_t tmem_base;
+  int abort_flag;
+};
+static_assert(sizeof(Bwd128Bars) <= 256, "barrier block");
+
+// A work item: one 128-key tile of one (sequence, head) and its live query tiles, from the
+// diagonal to the end of the tile's last document. Items are numbered key tile fastest.
+struct BwdItem {
+  int n, h, b, kv0, m_lo, nq;
+  long long seq0, vec0;
+};
+template <int BN, int BQ>
+__device__ __forceinline__ BwdItem bwd_item(const BwdParams& p, int it) {
+  BwdItem I;
+  I.n = it % p.nkt;
+  I.h = (it / p.nkt) % p.H;
+  I.b = it / (p.nkt * p.H);
+  I.seq0 = (long long)I.b * p.L;
+  I.kv0 = I.n * BN;
+  const int kv_last = min(I.kv0 + BN - 1, p.L - 1);
+  const int de_last = (int)(doc_end(p.offsets, p.n_offsets, I.seq0 + kv_last, I.seq0 + p.L) - I.seq0);
+  I.m_lo = I.kv0 / BQ;
+  I.nq = (de_last - 1) / BQ - I.m_lo + 1;
+  I.vec0 = ((long long)I.b * p.H + I.h) * p.L128;  // row 0 of this (b, h) in the padded vectors
+  return I;
+}
+
+}  // namespace ddattn

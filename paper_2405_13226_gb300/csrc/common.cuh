@@ -175,6 +175,8 @@ cudaError_t launch_attn_fwd(int d, const CUtensorMap& tq, const CUtensorMap& tk,
                             const FwdParams& p, cudaStream_t stream);
 cudaError_t launch_attn_bwd_main_d128(int d, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
                                       const CUtensorMap& tdo, const BwdParams& p, cudaStream_t stream);
+cudaError_t launch_attn_bwd_main_d128_persist(int d, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
+                                      const CUtensorMap& tdo, const BwdParams& p, cudaStream_t stream);
 cudaError_t launch_attn_bwd(int d, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
                             const CUtensorMap& tdo, const BwdParams& p, int phases, cudaStream_t stream);
 cudaError_t launch_rope_qk(const RopeParams& p, cudaStream_t stream);

@@ -50,6 +50,22 @@ def test_two_tile_forward_documents_on_pair_boundaries():
     print(errs)
 
 
+@pytest.mark.parametrize("d", [128, 80])
+def test_walking_backward_many_items_documents(d):
+    """Short sequences: the backward's CTAs each walk several key tiles (items) of
+    different sequences and step counts. 20 x 896 (7 key tiles: 280 items over one CTA
+    per SM, stride coprime with 7), documents of ragged lengths in every sequence."""
+    B, L = 20, 896
+    cuts = [0]
+    rng = np.random.RandomState(12)
+    for b in range(B):
+        inner = sorted(set(rng.randint(1, L, size=3).tolist()))
+        cuts += [b * L + x for x in inner] + [(b + 1) * L]
+    off = np.array(cuts, dtype=np.int32)
+    errs, _ = check_full(*_inputs(B, L, 2, d, seed=13), default_scale(d), off)
+    print(errs)
+
+
 @pytest.mark.parametrize("d", [64, 128])
 @pytest.mark.parametrize("seed", [0, 5])
 def test_document_mask_small(d, seed):
