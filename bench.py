@@ -59,7 +59,7 @@ def measured_traffic():
     vals = []
     for line in txt.splitlines():
         f = [x.strip() for x in line.split("|")]
-        if len(f) > 5 and f[2] == "attn_bwd_main_d128_kernel":
+        if len(f) > 5 and f[2] in ("attn_bwd_main_d128_kernel", "attn_bwd_main_d128_persist_kernel"):
             vals.append(float(f[5]))
     return sum(vals) / len(vals) if vals else None
 
@@ -336,7 +336,7 @@ def run_ours(args):
     # dominant kernel over the timed region: the backward main kernel
     main_ach = main_flops / (main_t * 1e-3) / 1e12
     peak = peaks["bf16_tflops_sustained"]
-    roofline = {"kernel": "attn_bwd_main_kernel<128>", "bound": "tensor", "achieved": main_ach, "peak": peak,
+    roofline = {"kernel": "attn_bwd_main (d=128: walking kernel for L <= 2048, per-key-tile kernel above)", "bound": "tensor", "achieved": main_ach, "peak": peak,
                 "unit": "TFLOP/s", "frac": main_ach / peak, "traffic": measured_traffic(),
                 "traffic_note": "mean dram__bytes_read+write per launch over the six buckets (ncu, "
                                 "profiles/attn_main_kernels_sweep_traffic.md); null if the kernel changed since",
