@@ -1,7 +1,10 @@
-// Causal / document-masked attention forward for sm_103a, two query tiles per CTA.
+// Causal / document-masked attention forward for sm_103a, two query tiles per work item.
 //
-// One CTA computes query tiles 2u and 2u + 1 (256 rows) of one (sequence,
-// head). Each key / value tile is loaded once for both. The two tiles have their
+// A work item is query tiles 2u and 2u + 1 (256 rows) of one (sequence, head); one CTA
+// per SM walks items (see attn_fwd_kernel), so that an item's loads overlap the previous
+// item's last softmax steps and epilogue and no CTA launch separates them (at L = 256
+// a one-item CTA spent ~2.6 of its ~9.2 us waiting for its first loads and ~0.9 on exit
+// and relaunch). Each key / value tile is loaded once for both tiles of an item. The two tiles have their
 // own softmax warpgroup, S buffer and O accumulator in TMEM, and the single
 // MMA-issuing thread alternates between them:
 //   ... PV_0(j-1), S_0(j), PV_1(j-1), S_1(j), PV_0(j), S_0(j+1) ...
@@ -21,8 +24,8 @@
 // producer with a plain arrive on k_empty (v_empty) of its ring stage. The
 // producers cannot wait on s_full themselves: with two ring stages the tensor
 // core may complete two phases of it before a producer looks, and a parity wait
-// cannot tell those apart. pv_done[t] is committed once, after the tile's last
-// PV, for the epilogue.
+// cannot tell those apart. pv_done[t] is committed once per item, after the
+// tile's last PV, for the epilogue.
 //
 // Warp roles (three warpgroups):
 //   WG0, WG1  softmax of tile 0 / tile 1: thread r owns query row r of its tile
@@ -30,9 +33,9 @@
 //             max and sum in the log2 domain with a lazy rescale of O (only when
 //             the running max grows by more than 8: P <= 256 stays exact enough
 //             in bf16 / fp32), P as bf16 pairs over the S buffer.
-//   WG2       warp 8: TMA producer for Q (both tiles, once) and the K ring, TMEM
-//             owner; warp 9: V ring producer; warp 10: the MMA issuer; warp 11
-//             idle. WG2 gives registers back (setmaxnreg.dec) to the softmax
+//   WG2       warp 8: K ring producer and TMEM owner; warp 9: V ring producer;
+//             warp 10: the MMA issuer; warp 11: Q producer (both tiles of each
+//             item). WG2 gives registers back (setmaxnreg.dec) to the softmax
 //             groups (setmaxnreg.inc).
 // MMA issue: the whole of warp 10 runs the issue loop (waits, descriptor
 // arithmetic) and one lane chosen by elect.sync issues each group of MMAs and
@@ -41,7 +44,7 @@
 // softmax warps, and the divergent form costs more instructions per MMA.
 // TMEM (512 columns): S_t at columns 128 t, O_t at 256 + 128 t.
 // Key tiles: tile t covers [lo_t, 2u + t] (lo_t: the key tile of the document
-// start of its first row); the CTA walks the union [lo_0, 2u + 1] and each
+// start of its first row); the item walks the union [lo_0, 2u + 1] and each
 // tile skips the key tiles outside its own range.
 #include "common.cuh"
 
@@ -72,7 +75,7 @@ static_assert(128 * FwdCfg<128>::REGS_LOW + 256 * FwdCfg<128>::REGS_HIGH <= 384 
 static_assert(128 * FwdCfg<64>::REGS_LOW + 256 * FwdCfg<64>::REGS_HIGH <= 384 * 168, "register split");
 
 struct FwdBars {
-  uint64_t q_full[2];
+  uint64_t q_full[2], q_empty[2];
   uint64_t k_full[2], k_empty[2], v_full[2], v_empty[2];
   uint64_t s_full[2], p_full[2], pv_done[2];
   uint64_t mma_drain;
@@ -82,6 +85,50 @@ struct FwdBars {
 static_assert(sizeof(FwdBars) <= 256, "barrier block");
 static_assert(FwdCfg<128>::KST == 2 && FwdCfg<128>::VST == 2, "ring barriers");
 
+// A work item: query tiles 2u and 2u + 1 of one (sequence, head). Items are numbered pair
+// fastest, heaviest pair (largest u) first.
+struct FwdItem {
+  int u, h, b;
+  long long seq0;
+  bool has1;              // an odd tile count leaves the last pair one tile
+  int lo0, lo1, hi0, hi1; // key-tile range [lo_t, hi_t] of tile t; lo_0 <= lo_1 (documents start in order)
+  int J0, NJ;             // the key tiles the item walks: J0 .. J0 + NJ - 1
+};
+__device__ __forceinline__ FwdItem fwd_item(const FwdParams& p, int it) {
+  constexpr int BM = 128, BN = 128;
+  const int nqp = (p.nqt + 1) >> 1;
+  FwdItem I;
+  I.u = nqp - 1 - it % nqp;
+  I.h = (it / nqp) % p.H;
+  I.b = it / (nqp * p.H);
+  I.seq0 = (long long)I.b * p.L;
+  I.has1 = 2 * I.u + 1 < p.nqt;
+  const int r1c = (2 * I.u + 1) * BM < p.L ? (2 * I.u + 1) * BM : p.L - 1;
+  I.lo0 = (int)(doc_start(p.offsets, p.n_offsets, I.seq0 + 2 * I.u * BM, I.seq0) - I.seq0) / BN;
+  I.lo1 = (int)(doc_start(p.offsets, p.n_offsets, I.seq0 + r1c, I.seq0) - I.seq0) / BN;
+  I.hi0 = 2 * I.u;
+  I.hi1 = 2 * I.u + 1;
+  I.J0 = I.lo0;
+  I.NJ = (I.has1 ? I.hi1 : I.hi0) - I.J0 + 1;
+  return I;
+}
+
+// A CTA per SM walks items c, c + G, c + 2G ... (G coprime with the pairs per sequence and
+// head, so every CTA meets every pair position), with the K / V rings, Q buffers and per-tile
+// barrier phases running on across items:
+//   * ring position jg counts the key tiles the CTA has loaded; stage jg % 2, parity
+//     (jg / 2) % 2, in every role;
+//   * Q_t of an item is loaded (by warp 11) once the previous item's last S_t has
+//     completed: the softmax thread that sees that S's commit relays it on q_empty[t];
+//   * the relays of K / V ring stages are those of one item, plus, after pv_done, the
+//     value tile whose last reader no S commit of the item covers: the item's last one,
+//     and tile 0's last one when tile 1's document starts at tile 1 (then tile 1 reads
+//     none of it);
+//   * an item's first PV into O_t needs no barrier of its own: it waits for that item's
+//     first p_full[t], which the tile's softmax group arrives only after its epilogue of
+//     the previous item has read O_t out.
+// A CPU discrete-event model of this protocol (random walks, random document starts,
+// random timings) runs in tests/test_fwd_walk_protocol.py.
 template <int D>
 __global__ void __launch_bounds__(384, 1)
     attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
@@ -94,23 +141,15 @@ __global__ void __launch_bounds__(384, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
   const int nqp = (p.nqt + 1) >> 1;
-  const int u = nqp - 1 - blockIdx.x;  // heaviest pairs first
-  const int h = blockIdx.y, b = blockIdx.z;
-  const long long seq0 = (long long)b * p.L;
-  const bool has1 = 2 * u + 1 < p.nqt;  // an odd tile count leaves the last pair one tile
-  // Key-tile range of each tile: [lo_t, hi_t]; lo_0 <= lo_1 (documents start in order).
-  const int r1c = (2 * u + 1) * C::BM < p.L ? (2 * u + 1) * C::BM : p.L - 1;
-  const int lo0 = (int)(doc_start(p.offsets, p.n_offsets, seq0 + 2 * u * C::BM, seq0) - seq0) / C::BN;
-  const int lo1 = (int)(doc_start(p.offsets, p.n_offsets, seq0 + r1c, seq0) - seq0) / C::BN;
-  const int hi0 = 2 * u, hi1 = 2 * u + 1;
-  const int J0 = lo0;
-  const int NJ = (has1 ? hi1 : hi0) - J0 + 1;  // key tiles walked by the CTA
+  const int n_items = nqp * p.H * p.B;
+  const int it_first = blockIdx.x, it_end = n_items, it_step = gridDim.x;
   Watchdog wd{&bars->abort_flag, p.status, p.timeout_ns};
 
   if (threadIdx.x == 0) {
     bars->abort_flag = 0;
     for (int t = 0; t < 2; t++) {
       mbar_init(&bars->q_full[t], 1);
+      mbar_init(&bars->q_empty[t], 1);
       mbar_init(&bars->s_full[t], 1);
       mbar_init(&bars->p_full[t], 128);
       mbar_init(&bars->pv_done[t], 1);
@@ -139,52 +178,55 @@ __global__ void __launch_bounds__(384, 1)
 
   if (wg == 2) {
   setmaxnreg_dec<C::REGS_LOW>();
-  if (warp == 8) {
-    // ---------------- Q (both tiles) + K producer
+  if (warp == 8 || warp == 9) {
+    // ---------------- K (warp 8) / V (warp 9) ring producer; jg = ring position
     if (lane == 0) {
-      prefetch_tmap(&tmQ);
-      prefetch_tmap(&tmK);
-      for (int t = 0; t < (has1 ? 2 : 1); t++) {
-        mbar_arrive_expect_tx(&bars->q_full[t], C::Q_BYTES);
-        for (int blk = 0; blk < C::DB; blk++)
-          tma_load_4d(sQ + t * C::Q_BYTES + blk * C::Q_BLK, &tmQ, &bars->q_full[t], 64 * blk, h,
-                      (2 * u + t) * C::BM, b);
-      }
-      int issued = 0;
-      for (int j = 0; j < NJ; j++) {
-        const int s = j % KST;
-        if (j >= KST && !mbar_wait(&bars->k_empty[s], ((j / KST) - 1) & 1, wd)) break;
-        mbar_arrive_expect_tx(&bars->k_full[s], C::KV_BYTES);
-        const int kv0 = (J0 + j) * C::BN;
-        for (int blk = 0; blk < C::DB; blk++)
-          tma_load_4d(sK + s * C::KV_BYTES + blk * C::KV_BLK, &tmK, &bars->k_full[s], 64 * blk, h, kv0, b);
-        if (j + C::PF < NJ)
-          for (int blk = 0; blk < C::DB; blk++) tma_prefetch_4d(&tmK, 64 * blk, h, kv0 + C::PF * C::BN, b);
-        issued = j + 1;
+      const bool isk = warp == 8;
+      const CUtensorMap* tm = isk ? &tmK : &tmV;
+      uint8_t* sR = isk ? sK : sV;
+      uint64_t* full = isk ? bars->k_full : bars->v_full;
+      uint64_t* empty = isk ? bars->k_empty : bars->v_empty;
+      prefetch_tmap(tm);
+      int jg = 0;
+      bool ok = true;
+      for (int it = it_first; ok && it < it_end; it += it_step) {
+        const FwdItem I = fwd_item(p, it);
+        for (int j = 0; j < I.NJ; j++, jg++) {
+          const int s = jg & 1;
+          if (jg >= KST && !(ok = mbar_wait(&empty[s], ((jg >> 1) - 1) & 1, wd))) break;
+          mbar_arrive_expect_tx(&full[s], C::KV_BYTES);
+          const int kv0 = (I.J0 + j) * C::BN;
+          for (int blk = 0; blk < C::DB; blk++)
+            tma_load_4d(sR + s * C::KV_BYTES + blk * C::KV_BLK, tm, &full[s], 64 * blk, I.h, kv0, I.b);
+          if (j + C::PF < I.NJ)
+            for (int blk = 0; blk < C::DB; blk++) tma_prefetch_4d(tm, 64 * blk, I.h, kv0 + C::PF * C::BN, I.b);
+        }
       }
       // Every copy lands before the CTA can exit (after an abort nobody else waits for them).
-      for (int t = 0; t < (has1 ? 2 : 1); t++) mbar_wait_drain(&bars->q_full[t], 0, wd.limit_ns);
-      for (int j = issued - KST < 0 ? 0 : issued - KST; j < issued; j++)
-        mbar_wait_drain(&bars->k_full[j % KST], (j / KST) & 1, wd.limit_ns);
+      for (int j = jg - KST < 0 ? 0 : jg - KST; j < jg; j++) mbar_wait_drain(&full[j & 1], (j >> 1) & 1, wd.limit_ns);
     }
-  } else if (warp == 9) {
-    // ---------------- V producer
+  } else if (warp == 11) {
+    // ---------------- Q producer: Q_t of an item once the previous one's last S_t is done
     if (lane == 0) {
-      prefetch_tmap(&tmV);
-      int issued = 0;
-      for (int j = 0; j < NJ; j++) {
-        const int s = j % VST;
-        if (j >= VST && !mbar_wait(&bars->v_empty[s], ((j / VST) - 1) & 1, wd)) break;
-        mbar_arrive_expect_tx(&bars->v_full[s], C::KV_BYTES);
-        const int kv0 = (J0 + j) * C::BN;
-        for (int blk = 0; blk < C::DB; blk++)
-          tma_load_4d(sV + s * C::KV_BYTES + blk * C::KV_BLK, &tmV, &bars->v_full[s], 64 * blk, h, kv0, b);
-        if (j + C::PF < NJ)
-          for (int blk = 0; blk < C::DB; blk++) tma_prefetch_4d(&tmV, 64 * blk, h, kv0 + C::PF * C::BN, b);
-        issued = j + 1;
+      prefetch_tmap(&tmQ);
+      int nload[2] = {0, 0};
+      bool ok = true;
+      for (int it = it_first; ok && it < it_end; it += it_step) {
+        const FwdItem I = fwd_item(p, it);
+#pragma unroll
+        for (int t = 0; t < 2; t++) {
+          if (!ok || !(t == 0 || I.has1)) continue;
+          if (nload[t] > 0 && !(ok = mbar_wait(&bars->q_empty[t], (nload[t] - 1) & 1, wd))) break;
+          mbar_arrive_expect_tx(&bars->q_full[t], C::Q_BYTES);
+          for (int blk = 0; blk < C::DB; blk++)
+            tma_load_4d(sQ + t * C::Q_BYTES + blk * C::Q_BLK, &tmQ, &bars->q_full[t], 64 * blk, I.h,
+                        (2 * I.u + t) * C::BM, I.b);
+          nload[t]++;
+        }
       }
-      for (int j = issued - VST < 0 ? 0 : issued - VST; j < issued; j++)
-        mbar_wait_drain(&bars->v_full[j % VST], (j / VST) & 1, wd.limit_ns);
+#pragma unroll
+      for (int t = 0; t < 2; t++)
+        if (nload[t] > 0) mbar_wait_drain(&bars->q_full[t], (nload[t] - 1) & 1, wd.limit_ns);
     }
   } else if (warp == 10) {
     // ---------------- MMA issuer: the whole warp runs the loop, one elected lane issues
@@ -196,8 +238,16 @@ __global__ void __launch_bounds__(384, 1)
       const uint64_t dQ0 = sdesc_sw128(smem_u32(sQ), 16, 1024);
       const uint64_t dK0 = sdesc_sw128(smem_u32(sK), 16, 1024);
       const uint64_t dV0 = sdesc_sw128(smem_u32(sV), C::KV_BLK, 1024);
-      int ns[2] = {0, 0}, npv[2] = {0, 0};  // S and PV issued per tile (static indices only)
+      // Running counts (static indices only): PV issued per tile, items per tile; per item:
+      // S and PV issued per tile.
+      int npv[2] = {0, 0}, nit[2] = {0, 0};
+      int jg0 = 0;
       bool ok = true;
+      for (int it = it_first; ok && it < it_end; it += it_step) {
+      const FwdItem I = fwd_item(p, it);
+      const bool has1 = I.has1;
+      const int lo0 = I.lo0, lo1 = I.lo1, hi0 = I.hi0, hi1 = I.hi1, J0 = I.J0, NJ = I.NJ;
+      int ns_i[2] = {0, 0}, npv_i[2] = {0, 0};
       for (int j = 0; j <= NJ && ok; j++) {
         const int kt = J0 + j;
 #pragma unroll
@@ -206,12 +256,12 @@ __global__ void __launch_bounds__(384, 1)
           const int lo_t = t ? lo1 : lo0, hi_t = t ? hi1 : hi0;
           // O_t += P_t V_{j-1}
           if (ok && tile && j >= 1 && kt - 1 >= lo_t && kt - 1 <= hi_t) {
-            const int i = j - 1, vs = i % VST;
-            ok = __all_sync(0xffffffffu, mbar_wait(&bars->v_full[vs], (i / VST) & 1, wd) &&
+            const int jv = jg0 + j - 1;
+            ok = __all_sync(0xffffffffu, mbar_wait(&bars->v_full[jv & 1], (jv >> 1) & 1, wd) &&
                                              mbar_wait(&bars->p_full[t], npv[t] & 1, wd));
           }
           if (ok && tile && j >= 1 && kt - 1 >= lo_t && kt - 1 <= hi_t) {
-            const int i = j - 1, vs = i % VST;
+            const int vs = (jg0 + j - 1) & 1;
             tc_fence_after();
             const uint64_t dV = dV0 + ((uint32_t)(vs * C::KV_BYTES) >> 4);
             const uint32_t tP = tmem + C::TMEM_S + t * 128;
@@ -219,20 +269,21 @@ __global__ void __launch_bounds__(384, 1)
 #pragma unroll
               for (int kk = 0; kk < C::BN / 16; kk++)
                 umma_bf16_ts(tmem + C::TMEM_O + t * 128, tP + kk * 8, dV + (uint32_t)((kk * 2048) >> 4), idesc_o,
-                             (npv[t] > 0 || kk > 0) ? 1u : 0u);
+                             (npv_i[t] > 0 || kk > 0) ? 1u : 0u);
               if (kt - 1 == hi_t) umma_commit(&bars->pv_done[t]);  // the tile's last PV: for the epilogue
             }
             __syncwarp();
             npv[t]++;
+            npv_i[t]++;
           }
           // S_t = Q_t K_j^T into the buffer PV_t has just read (issue order keeps them apart)
           if (ok && tile && j < NJ && kt >= lo_t && kt <= hi_t) {
-            const int ks = j % KST;
-            ok = __all_sync(0xffffffffu, mbar_wait(&bars->k_full[ks], (j / KST) & 1, wd) &&
-                                             (ns[t] > 0 || mbar_wait(&bars->q_full[t], 0, wd)));
+            const int jk = jg0 + j;
+            ok = __all_sync(0xffffffffu, mbar_wait(&bars->k_full[jk & 1], (jk >> 1) & 1, wd) &&
+                                             (ns_i[t] > 0 || mbar_wait(&bars->q_full[t], nit[t] & 1, wd)));
           }
           if (ok && tile && j < NJ && kt >= lo_t && kt <= hi_t) {
-            const int ks = j % KST;
+            const int ks = (jg0 + j) & 1;
             tc_fence_after();
             const uint64_t dQ = dQ0 + ((uint32_t)(t * C::Q_BYTES) >> 4);
             const uint64_t dK = dK0 + ((uint32_t)(ks * C::KV_BYTES) >> 4);
@@ -247,9 +298,13 @@ __global__ void __launch_bounds__(384, 1)
               umma_commit(&bars->s_full[t]);
             }
             __syncwarp();
-            ns[t]++;
+            ns_i[t]++;
           }
         }
+      }
+      nit[0]++;
+      if (has1) nit[1]++;
+      jg0 += NJ;
       }
       if (leader) umma_commit(&bars->mma_drain);
       __syncwarp();
@@ -261,28 +316,40 @@ __global__ void __launch_bounds__(384, 1)
   // ---------------- softmax of tile t = wg: thread r <-> query row r <-> TMEM lane r
   const int t = wg;
   const int r = threadIdx.x & 127;
-  const int row0 = (2 * u + t) * C::BM;
-  const int row = row0 + r;
-  const int rowc = row < p.L ? row : p.L - 1;
-  const int lo_t = t ? lo1 : lo0;
-  const int nt = (t == 0 || has1) ? (t ? hi1 : hi0) - lo_t + 1 : 0;
-  const int ds = (int)(doc_start(p.offsets, p.n_offsets, seq0 + rowc, seq0) - seq0);
   const uint32_t tl = tmem + ((uint32_t)((warp & 3) * 32) << 16);
   const uint32_t sbuf = tl + C::TMEM_S + t * 128;
   const uint32_t obuf = tl + C::TMEM_O + t * 128;
   const float sl2 = p.scale_log2;
   const uint64_t sl2x2 = f32x2(sl2, sl2);
-  float m_run = -INFINITY, l_run = 0.f;
+  int jg0 = 0, nit = 0, ns = 0;  // ring position of the item's first key tile, items of this tile, S seen
   bool ok = true;
+  for (int it = it_first; ok && it < it_end; it += it_step) {
+  const FwdItem I = fwd_item(p, it);
+  if (!(t == 0 || I.has1)) {
+    jg0 += I.NJ;
+    continue;
+  }
+  const bool has1 = I.has1;
+  const int lo1 = I.lo1, J0 = I.J0, h = I.h, b = I.b;
+  const long long seq0 = I.seq0;
+  const int row0 = (2 * I.u + t) * C::BM;
+  const int row = row0 + r;
+  const int rowc = row < p.L ? row : p.L - 1;
+  const int lo_t = t ? I.lo1 : I.lo0, hi_t = t ? I.hi1 : I.hi0;
+  const int nt = hi_t - lo_t + 1;
+  const int ds = (int)(doc_start(p.offsets, p.n_offsets, seq0 + rowc, seq0) - seq0);
+  float m_run = -INFINITY, l_run = 0.f;
   for (int i = 0; i < nt && ok; i++) {
     const int kv0 = (lo_t + i) * C::BN;
-    ok = __all_sync(0xffffffffu, mbar_wait(&bars->s_full[t], i & 1, wd));
+    ok = __all_sync(0xffffffffu, mbar_wait(&bars->s_full[t], ns & 1, wd));
     if (!ok) break;
+    ns++;
     tc_fence_after();
     if (r == 0) {  // relay: this tile is the last reader of key tile kt / value tile kt - 1
-      const int kt = lo_t + i;
-      if (t == 1 || !(has1 && kt >= lo1)) mbar_arrive(&bars->k_empty[(kt - J0) & 1]);
-      if (i >= 1 && (t == 1 || !(has1 && kt - 1 >= lo1))) mbar_arrive(&bars->v_empty[(kt - 1 - J0) & 1]);
+      const int kt = lo_t + i, jk = jg0 + kt - J0;
+      if (t == 1 || !(has1 && kt >= lo1)) mbar_arrive(&bars->k_empty[jk & 1]);
+      if (i >= 1 && (t == 1 || !(has1 && kt - 1 >= lo1))) mbar_arrive(&bars->v_empty[(jk - 1) & 1]);
+      if (i == nt - 1) mbar_arrive(&bars->q_empty[t]);  // the tile's last S is done: Q_t may be replaced
     }
     uint32_t v0[32], v1[32], v2[32], v3[32];
     tmem_ld32(sbuf + 0, v0);
@@ -353,9 +420,14 @@ __global__ void __launch_bounds__(384, 1)
     mbar_arrive(&bars->p_full[t]);
   }
   // Epilogue: O / l -> bf16, LSE = (m + log2 l) * ln2.
-  if (ok && nt > 0) ok = __all_sync(0xffffffffu, mbar_wait(&bars->pv_done[t], 0, wd));
-  if (ok && nt > 0) {
+  if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&bars->pv_done[t], nit & 1, wd));
+  if (ok) {
     tc_fence_after();
+    // The value tile whose last reader no S commit of the item covers: the item's last
+    // one (tile 1's, or tile 0's without a tile 1), and tile 0's last one when tile 1's
+    // document starts at tile 1 (tile 1 reads none of it).
+    if (r == 0 && (t == (has1 ? 1 : 0) || (t == 0 && has1 && lo1 > I.hi0)))
+      mbar_arrive(&bars->v_empty[(jg0 + hi_t - J0) & 1]);
     const float inv_l = l_run > 0.f ? 1.f / l_run : 0.f;
     const float m_use = (m_run == -INFINITY) ? 0.f : m_run;
     __nv_bfloat16* orow = p.o + (((long long)b * p.L + rowc) * p.H + h) * D;
@@ -382,6 +454,9 @@ __global__ void __launch_bounds__(384, 1)
     if (row < p.L)
       p.lse[((long long)b * p.H + h) * p.L + row] = l_run > 0.f ? (m_use + __log2f(l_run)) * kLn2 : -INFINITY;
   }
+  nit++;
+  jg0 += I.NJ;
+  }
   }
 
   tc_fence_before();
@@ -397,14 +472,32 @@ static cudaError_t launch_fwd_d(const CUtensorMap& tq, const CUtensorMap& tk, co
                                const FwdParams& p, cudaStream_t stream) {
   using C = FwdCfg<D>;
   static bool attr_set = false;
+  static int nsm = 0;
   if (!attr_set) {
     cudaError_t e =
         cudaFuncSetAttribute(attn_fwd_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_BYTES);
     if (e != cudaSuccess) return e;
+    int dev = 0;
+    if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+    if ((e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
+    if (nsm < 1) nsm = 1;
     attr_set = true;
   }
-  dim3 grid((p.nqt + 1) / 2, p.H, p.B);
-  attn_fwd_kernel<D><<<grid, C::THREADS, C::SMEM_BYTES, stream>>>(tq, tk, tv, p);
+  // One CTA per SM (shared memory allows no more) walking items; a stride coprime with the
+  // pairs per (sequence, head) gives every CTA every pair position (their key-tile counts differ).
+  const int nqp = (p.nqt + 1) / 2;
+  const long long items = (long long)nqp * p.H * p.B;
+  long long G = items < nsm ? items : nsm;
+  auto gcd = [](long long x, long long y) {
+    while (y) {
+      const long long t = x % y;
+      x = y;
+      y = t;
+    }
+    return x;
+  };
+  while (G > 1 && gcd(G, nqp) != 1) G--;
+  attn_fwd_kernel<D><<<(unsigned)G, C::THREADS, C::SMEM_BYTES, stream>>>(tq, tk, tv, p);
   return cudaGetLastError();
 }
 
