@@ -193,6 +193,7 @@ dd_status dd_attn_fwd(const dd_attn_desc* desc, const void* q, const void* k, co
   p.o = static_cast<__nv_bfloat16*>(o);
   p.lse = lse;
   p.status = static_cast<int*>(ws);
+  p.work_ctr = reinterpret_cast<unsigned int*>(static_cast<uint8_t*>(ws) + 64);  // inside the status block
   p.timeout_ns = wait_limit_ns();
   cudaError_t e = launch_attn_fwd(desc->d, tq, tk, tv, p, static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? DD_OK : DD_ERR_CUDA;

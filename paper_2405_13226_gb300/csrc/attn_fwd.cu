@@ -74,7 +74,14 @@ struct FwdCfg {
 static_assert(128 * FwdCfg<128>::REGS_LOW + 256 * FwdCfg<128>::REGS_HIGH <= 384 * 168, "register split");
 static_assert(128 * FwdCfg<64>::REGS_LOW + 256 * FwdCfg<64>::REGS_HIGH <= 384 * 168, "register split");
 
+// The item ring: warp 11 claims each next item and publishes its index to the roles that
+// read it: the K and V producer lanes, the 32 lanes of the MMA warp and the 256 softmax
+// threads, each of which arrives on item_empty after reading.
+constexpr int kItemRing = 4, kItemReaders = 1 + 1 + 32 + 256;
+
 struct FwdBars {
+  uint64_t item_full[kItemRing], item_empty[kItemRing];
+  int item[kItemRing];  // -1: no more items
   uint64_t q_full[2], q_empty[2];
   uint64_t k_full[2], k_empty[2], v_full[2], v_empty[2];
   uint64_t s_full[2], p_full[2], pv_done[2];
@@ -113,9 +120,15 @@ __device__ __forceinline__ FwdItem fwd_item(const FwdParams& p, int it) {
   return I;
 }
 
-// A CTA per SM walks items c, c + G, c + 2G ... (G coprime with the pairs per sequence and
-// head, so every CTA meets every pair position), with the K / V rings, Q buffers and per-tile
-// barrier phases running on across items:
+// A CTA per SM walks items, starting with item blockIdx.x. Without a document mask the next
+// is item + G (G coprime with the pairs per sequence and head, so every CTA meets every pair
+// position and the costs even out; the CTAs on one sequence's pairs share its K / V tiles in
+// L2). With a document mask the item costs vary with the documents: each next item is
+// claimed from a global counter (item G + count) when the CTA starts loading the previous
+// one, so the items spread over the CTAs as they free up. Over four DM steps (8 x 8192)
+// static assignment was 8-10% slower than one CTA per item, claiming within 0-4%; over the
+// plain buckets claiming was 2% slower than static at L = 1024 and 8192. The K / V
+// rings, Q buffers and per-tile barrier phases run on across items:
 //   * ring position jg counts the key tiles the CTA has loaded; stage jg % 2, parity
 //     (jg / 2) % 2, in every role;
 //   * Q_t of an item is loaded (by warp 11) once the previous item's last S_t has
@@ -129,6 +142,17 @@ __device__ __forceinline__ FwdItem fwd_item(const FwdParams& p, int it) {
 //     the previous item has read O_t out.
 // A CPU discrete-event model of this protocol (random walks, random document starts,
 // random timings) runs in tests/test_fwd_walk_protocol.py.
+// The n-th item of a CTA from its item ring, for a role whose whole warp waits (-1: no
+// more items, or the CTA was aborted: then ok is false).
+__device__ __forceinline__ int fwd_next_item(FwdBars* bars, int n, bool& ok, const Watchdog& wd) {
+  const int slot = n & (kItemRing - 1);
+  ok = __all_sync(0xffffffffu, ok && mbar_wait(&bars->item_full[slot], (n / kItemRing) & 1, wd));
+  if (!ok) return -1;
+  const int it = *reinterpret_cast<volatile int*>(&bars->item[slot]);
+  mbar_arrive(&bars->item_empty[slot]);
+  return it;
+}
+
 template <int D>
 __global__ void __launch_bounds__(384, 1)
     attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
@@ -142,11 +166,14 @@ __global__ void __launch_bounds__(384, 1)
 
   const int nqp = (p.nqt + 1) >> 1;
   const int n_items = nqp * p.H * p.B;
-  const int it_first = blockIdx.x, it_end = n_items, it_step = gridDim.x;
   Watchdog wd{&bars->abort_flag, p.status, p.timeout_ns};
 
   if (threadIdx.x == 0) {
     bars->abort_flag = 0;
+    for (int i = 0; i < kItemRing; i++) {
+      mbar_init(&bars->item_full[i], 1);
+      mbar_init(&bars->item_empty[i], kItemReaders);
+    }
     for (int t = 0; t < 2; t++) {
       mbar_init(&bars->q_full[t], 1);
       mbar_init(&bars->q_empty[t], 1);
@@ -189,7 +216,12 @@ __global__ void __launch_bounds__(384, 1)
       prefetch_tmap(tm);
       int jg = 0;
       bool ok = true;
-      for (int it = it_first; ok && it < it_end; it += it_step) {
+      for (int n = 0; ok; n++) {
+        const int slot = n & (kItemRing - 1);
+        if (!(ok = mbar_wait(&bars->item_full[slot], (n / kItemRing) & 1, wd))) break;
+        const int it = *reinterpret_cast<volatile int*>(&bars->item[slot]);
+        mbar_arrive(&bars->item_empty[slot]);
+        if (it < 0) break;
         const FwdItem I = fwd_item(p, it);
         for (int j = 0; j < I.NJ; j++, jg++) {
           const int s = jg & 1;
@@ -211,7 +243,13 @@ __global__ void __launch_bounds__(384, 1)
       prefetch_tmap(&tmQ);
       int nload[2] = {0, 0};
       bool ok = true;
-      for (int it = it_first; ok && it < it_end; it += it_step) {
+      int it = blockIdx.x;
+      for (int n = 0; ok; n++) {
+        const int slot = n & (kItemRing - 1);
+        if (n >= kItemRing && !(ok = mbar_wait(&bars->item_empty[slot], ((n / kItemRing) - 1) & 1, wd))) break;
+        *reinterpret_cast<volatile int*>(&bars->item[slot]) = it < n_items ? it : -1;
+        mbar_arrive(&bars->item_full[slot]);  // release: the index is visible to the waiting roles
+        if (it >= n_items) break;
         const FwdItem I = fwd_item(p, it);
 #pragma unroll
         for (int t = 0; t < 2; t++) {
@@ -223,6 +261,7 @@ __global__ void __launch_bounds__(384, 1)
                         (2 * I.u + t) * C::BM, I.b);
           nload[t]++;
         }
+        it = p.offsets ? (int)gridDim.x + (int)atomicAdd(p.work_ctr, 1u) : it + (int)gridDim.x;
       }
 #pragma unroll
       for (int t = 0; t < 2; t++)
@@ -243,7 +282,9 @@ __global__ void __launch_bounds__(384, 1)
       int npv[2] = {0, 0}, nit[2] = {0, 0};
       int jg0 = 0;
       bool ok = true;
-      for (int it = it_first; ok && it < it_end; it += it_step) {
+      for (int n = 0; ok; n++) {
+      const int it = fwd_next_item(bars, n, ok, wd);
+      if (it < 0) break;
       const FwdItem I = fwd_item(p, it);
       const bool has1 = I.has1;
       const int lo0 = I.lo0, lo1 = I.lo1, hi0 = I.hi0, hi1 = I.hi1, J0 = I.J0, NJ = I.NJ;
@@ -323,7 +364,9 @@ __global__ void __launch_bounds__(384, 1)
   const uint64_t sl2x2 = f32x2(sl2, sl2);
   int jg0 = 0, nit = 0, ns = 0;  // ring position of the item's first key tile, items of this tile, S seen
   bool ok = true;
-  for (int it = it_first; ok && it < it_end; it += it_step) {
+  for (int n = 0; ok; n++) {
+  const int it = fwd_next_item(bars, n, ok, wd);
+  if (it < 0) break;
   const FwdItem I = fwd_item(p, it);
   if (!(t == 0 || I.has1)) {
     jg0 += I.NJ;
@@ -497,6 +540,10 @@ static cudaError_t launch_fwd_d(const CUtensorMap& tq, const CUtensorMap& tk, co
     return x;
   };
   while (G > 1 && gcd(G, nqp) != 1) G--;
+  if (p.offsets) {  // the claim counter of the document-masked walk
+    cudaError_t e = cudaMemsetAsync(p.work_ctr, 0, sizeof(unsigned int), stream);
+    if (e != cudaSuccess) return e;
+  }
   attn_fwd_kernel<D><<<(unsigned)G, C::THREADS, C::SMEM_BYTES, stream>>>(tq, tk, tv, p);
   return cudaGetLastError();
 }

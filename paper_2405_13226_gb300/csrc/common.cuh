@@ -136,6 +136,7 @@ struct FwdParams {
   __nv_bfloat16* o;
   float* lse;
   int* status;
+  unsigned int* work_ctr;  // items claimed past the first G (in the workspace's status block, zeroed per launch)
   unsigned long long timeout_ns;
 };
 

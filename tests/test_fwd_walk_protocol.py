@@ -4,8 +4,10 @@ in which one CTA per SM computes several query-tile pairs in turn).
 Per CTA: a Q producer, a K producer, a V producer, the MMA issuer and two softmax
 groups, synchronised by mbarriers with parity waits; copies land after random delays
 and the tensor core runs MMAs in issue order, each commit arriving once everything
-issued before it has completed. Across the items (query-tile pairs of any sequence) a
-CTA walks:
+issued before it has completed. The Q producer claims the CTA's items one at a time and
+publishes each through a 4-slot ring in shared memory (item_full, item_empty with one
+arrival per reading role), closed by an end marker; every other role takes its items
+from that ring. Across the items (query-tile pairs of any sequence) a CTA walks:
   * the K / V rings continue with a running ring index;
   * Q of tile t is reloaded once the last S of tile t of the previous item has completed:
     the softmax thread that sees that S's commit relays it (q_empty);
@@ -82,11 +84,19 @@ def tiles(it):
     return (0, 1) if it["has1"] else (0,)
 
 
+N_READERS = 5     # K producer, V producer, MMA issuer, two softmax groups
+RING = 4
+
+
 def simulate_walk(items, seed, tile0_v_relay=True, q_empty_wait=True):
     rnd = random.Random(seed)
     names = ["q0", "q1", "k0", "k1", "v0", "v1", "s0", "s1", "pv0", "pv1", "drain",
              "qe0", "qe1", "ke0", "ke1", "ve0", "ve1"]
     bars = {n: Barrier() for n in names}
+    for i in range(RING):
+        bars["if%d" % i] = Barrier()
+        bars["ie%d" % i] = Barrier(N_READERS)
+    ring = [None] * RING
     bars["p0"], bars["p1"] = Barrier(), Barrier()       # one arrival per softmax group in the model
     now = [0]
     events = []
@@ -121,19 +131,41 @@ def simulate_walk(items, seed, tile0_v_relay=True, q_empty_wait=True):
             else:
                 events.append((busy_until[0] + 1, lambda b=arg: bars[b].arrive()))
 
+    def publish(n, value):
+        slot = n % RING
+        if n >= RING:
+            yield ("wait", "ie%d" % slot, ((n // RING) - 1) & 1)
+        ring[slot] = value
+        bars["if%d" % slot].arrive()
+
+    def take(n):
+        """A reading role's n-th item from the ring (None: the end marker)."""
+        slot = n % RING
+        yield ("wait", "if%d" % slot, (n // RING) & 1)
+        value = ring[slot]
+        bars["ie%d" % slot].arrive()
+        return value
+
     def q_producer():
         n_t = [0, 0]
-        for it in items:
+        for n, it in enumerate(items):
+            yield from publish(n, it)
             for t in tiles(it):
                 if n_t[t] > 0 and q_empty_wait:
                     yield ("wait", "qe%d" % t, (n_t[t] - 1) & 1)
                 bars["q%d" % t].expect_tx(1)
                 copy("q%d" % t, ("q", t))
                 n_t[t] += 1
+        yield from publish(len(items), None)
 
     def ring_producer(kind):
         jg = 0
-        for it in items:
+        n_item = 0
+        while True:
+            it = yield from take(n_item)
+            if it is None:
+                break
+            n_item += 1
             for j in range(it["NJ"]):
                 s = jg & 1
                 if jg >= 2:
@@ -146,7 +178,12 @@ def simulate_walk(items, seed, tile0_v_relay=True, q_empty_wait=True):
         jg0 = 0
         n_t = [0, 0]            # items with tile t so far
         ns, npv = [0, 0], [0, 0]
-        for it in items:
+        n_item = 0
+        while True:
+            it = yield from take(n_item)
+            if it is None:
+                break
+            n_item += 1
             first_pv, first_s = [True, True], [True, True]
             for j in range(it["NJ"] + 1):
                 kt = it["J0"] + j
@@ -180,7 +217,12 @@ def simulate_walk(items, seed, tile0_v_relay=True, q_empty_wait=True):
         jg0 = 0
         n_t = 0
         ns = 0
-        for it in items:
+        n_item = 0
+        while True:
+            it = yield from take(n_item)
+            if it is None:
+                break
+            n_item += 1
             if t in tiles(it):
                 lo_t, hi_t = (it["lo1"], it["hi1"]) if t else (it["lo0"], it["hi0"])
                 nt = hi_t - lo_t + 1
@@ -317,3 +359,4 @@ def test_walk_protocol_negative_controls():
             except (Hazard, OverArrival):
                 caught += 1
     assert caught > 0
+
