@@ -120,14 +120,13 @@ __device__ __forceinline__ FwdItem fwd_item(const FwdParams& p, int it) {
   return I;
 }
 
-// A CTA per SM walks items, starting with item blockIdx.x. Without a document mask the next
-// is item + G (G coprime with the pairs per sequence and head, so every CTA meets every pair
-// position and the costs even out; the CTAs on one sequence's pairs share its K / V tiles in
-// L2). With a document mask the item costs vary with the documents: each next item is
-// claimed from a global counter (item G + count) when the CTA starts loading the previous
-// one, so the items spread over the CTAs as they free up. Over four DM steps (8 x 8192)
-// static assignment was 8-10% slower than one CTA per item, claiming within 0-4%; over the
-// plain buckets claiming was 2% slower than static at L = 1024 and 8192. The K / V
+// A CTA per SM walks items, starting with item blockIdx.x; each next item is claimed from a
+// global counter (item G + count) when the CTA starts loading the previous one, so items
+// spread over the CTAs as they free up, whatever their cost (with document masks it varies
+// with the documents). Items are numbered sequence and head slowest, so the CTAs working at
+// one time share each sequence's K / V tiles in L2. Over four DM steps (8 x 8192) a static
+// assignment (items c, c + G, ...) was 8-10% slower than one CTA per item and claiming
+// 0-4%; over the plain buckets claiming was within 0-2% of static. The K / V
 // rings, Q buffers and per-tile barrier phases run on across items:
 //   * ring position jg counts the key tiles the CTA has loaded; stage jg % 2, parity
 //     (jg / 2) % 2, in every role;
@@ -261,7 +260,7 @@ __global__ void __launch_bounds__(384, 1)
                         (2 * I.u + t) * C::BM, I.b);
           nload[t]++;
         }
-        it = p.offsets ? (int)gridDim.x + (int)atomicAdd(p.work_ctr, 1u) : it + (int)gridDim.x;
+        it = (int)gridDim.x + (int)atomicAdd(p.work_ctr, 1u);
       }
 #pragma unroll
       for (int t = 0; t < 2; t++)
@@ -540,10 +539,8 @@ static cudaError_t launch_fwd_d(const CUtensorMap& tq, const CUtensorMap& tk, co
     return x;
   };
   while (G > 1 && gcd(G, nqp) != 1) G--;
-  if (p.offsets) {  // the claim counter of the document-masked walk
-    cudaError_t e = cudaMemsetAsync(p.work_ctr, 0, sizeof(unsigned int), stream);
-    if (e != cudaSuccess) return e;
-  }
+  cudaError_t e = cudaMemsetAsync(p.work_ctr, 0, sizeof(unsigned int), stream);  // the claim counter
+  if (e != cudaSuccess) return e;
   attn_fwd_kernel<D><<<(unsigned)G, C::THREADS, C::SMEM_BYTES, stream>>>(tq, tk, tv, p);
   return cudaGetLastError();
 }
