@@ -1,10 +1,12 @@
-"""CPU model of the forward kernel's barrier protocol (csrc/attn_fwd.cu).
+"""CPU model of the forward kernel's per-item barrier protocol (csrc/attn_fwd.cu): one
+work item (two query tiles) on its own. tests/test_fwd_walk_protocol.py models the walk
+over many items that the kernel runs; this file keeps the single-item cases exhaustive
+and the negative control of the first design.
 
-One CTA computes two query tiles; a K producer, a V producer, the MMA issuer
-and two softmax groups synchronise through mbarriers with parity waits, and
-the K / V ring stages are handed back to the producers by the softmax thread
-that last read a key tile (k_empty / v_empty arrivals relayed after it has seen
-the s_full commit of the S that followed the tile's last use). The model runs
+A K producer, a V producer, the MMA issuer and two softmax groups synchronise through
+mbarriers with parity waits, and the K / V ring stages are handed back to the producers
+by the softmax thread that last read a key tile (k_empty / v_empty arrivals relayed after
+it has seen the s_full commit of the S that followed the tile's last use). The model runs
 those agents as coroutines against barrier objects with the hardware's parity
 semantics, an in-order tensor pipe and copies that land after random delays,
 and checks, for every query-tile pair and document-start placement up to 17

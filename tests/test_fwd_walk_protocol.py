@@ -360,3 +360,38 @@ def test_walk_protocol_negative_controls():
                 caught += 1
     assert caught > 0
 
+
+
+def items_from_offsets(offsets, B, L):
+    """The forward's work items of a document-masked batch: per sequence b and pair u, the
+    key-tile ranges from the document starts of the pair's first rows (as the kernel
+    derives them from cu_doc_offsets)."""
+    import bisect
+    nqt = (L + 127) // 128
+    out = []
+    for b in range(B):
+        seq0 = b * L
+
+        def doc_start(row):
+            t = seq0 + row
+            i = bisect.bisect_right(offsets, t) - 1
+            return max(offsets[i], seq0) - seq0 if i >= 0 else 0
+
+        for u in range((nqt + 1) // 2 - 1, -1, -1):
+            r1 = min((2 * u + 1) * 128, L - 1)
+            out.append(make_item(nqt, u, doc_start(2 * u * 128) // 128, doc_start(r1) // 128))
+    return out
+
+
+@pytest.mark.parametrize("kind", ["dm", "pack"])
+def test_walk_protocol_on_document_masked_batches(kind):
+    """Items of the DM and Pack-8k steps the benchmark times (8 x 8192), walked in the
+    orders a CTA meets them: runs of consecutive claims and strided picks."""
+    from paper_2405_13226_gb300 import workloads as wl
+    for seed in range(2):
+        off = (wl.concat_and_chunk_offsets(seed) if kind == "dm" else wl.packed_dm_offsets(seed)).tolist()
+        items = items_from_offsets(off, 8, 8192)
+        rnd = random.Random(seed)
+        for start in rnd.sample(range(len(items) - 6), 4):
+            simulate_walk(items[start:start + 6], seed)
+        simulate_walk(items[seed::37][:6], seed + 1)
