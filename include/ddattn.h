@@ -39,10 +39,14 @@
  *                                last B*L. Sequence boundaries b*L always cut
  *                                documents, listed or not. NULL = plain causal.
  *   ws                         : workspace of dd_attn_workspace_size() bytes,
- *                                256-byte aligned. Its first 16 bytes hold the
- *                                device status word: zero it once before first
- *                                use (dd_attn_clear_status). fwd and bwd may
- *                                share one workspace sized for bwd.
+ *                                256-byte aligned. Its first 256 bytes are a
+ *                                status block: the device status word in the
+ *                                first 16 bytes (zero it once before first use,
+ *                                dd_attn_clear_status) and the forward's
+ *                                work-item counter at byte 64 (each forward call
+ *                                zeroes it on its stream). fwd and bwd may share
+ *                                one workspace sized for bwd; calls that share a
+ *                                workspace must not overlap on the GPU.
  * All data pointers must be 16-byte aligned. Calls are asynchronous and
  * ordered on `stream` (a cudaStream_t; NULL = legacy default stream).
  *
@@ -93,7 +97,10 @@ typedef struct {
  * L) * d/2 pairs). Returns 0 for an invalid descriptor. */
 size_t dd_attn_workspace_size(const dd_attn_desc* desc, int for_bwd);
 
-/* Forward (Sec. 2.2 step; mask per cu_doc_offsets): writes o and lse. */
+/* Forward (Sec. 2.2 step; mask per cu_doc_offsets): writes o and lse. One CTA
+ * per SM walks the work items (two 128-row query tiles of one sequence and
+ * head), claiming each next one from the counter in the workspace's status
+ * block; a memset of that counter precedes the kernel on `stream`. */
 dd_status dd_attn_fwd(const dd_attn_desc* desc, const void* q, const void* k, const void* v, void* o, float* lse,
                       void* ws, size_t ws_bytes, void* stream);
 
