@@ -540,25 +540,18 @@ template <int D>
 static cudaError_t launch_bwd_d(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
                                 const CUtensorMap& tdo, const BwdParams& p, int phases, cudaStream_t stream) {
   using C = BwdCfg<D>;
-  if constexpr (D == 64) {
-    static bool attr_set = false;
-    if (!attr_set) {
-      cudaError_t e =
-          cudaFuncSetAttribute(attn_bwd_main_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_BYTES);
-      if (e != cudaSuccess) return e;
-      attr_set = true;
-    }
-  }
-  static int nsm = 0;
-  if (!nsm) {
-    int dev = 0;
-    cudaGetDevice(&dev);
-    cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
-    if (nsm < 1) nsm = 152;
-  }
+  static int nsm_dev[kMaxDevices] = {};
+  int nsm = 0;
+  // d = 64 has its own main kernel (its shared memory set here); the pre / post kernels use
+  // none, and the d = 80 / 128 main kernels are set up by their launchers.
+  cudaError_t e;
+  if constexpr (D == 64)
+    e = kernel_setup(nsm_dev, attn_bwd_main_kernel<D>, C::SMEM_BYTES, &nsm);
+  else
+    e = kernel_setup(nsm_dev, attn_bwd_pre_kernel<D>, 0, &nsm);
+  if (e != cudaSuccess) return e;
   const long long work = (long long)p.B * p.L * p.H * (D / 8);
   const int ew_blocks = (int)std::min<long long>((work + 255) / 256, (long long)nsm * 8);
-  cudaError_t e = cudaSuccess;
   if (phases & 1) {
     if (p.rope_tab && (e = launch_rope_table(p.L, D, p.rope, p.rope_tab, p.rope_tab_rows, stream)) != cudaSuccess)
       return e;

@@ -463,13 +463,10 @@ template <int DH>
 static cudaError_t launch_big(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
                               const CUtensorMap& tdo, const BwdParams& p, cudaStream_t stream) {
   using C = BwdBig<DH>;
-  static bool attr_set = false;
-  if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(attn_bwd_main_d128_kernel<DH>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         C::SMEM_BYTES);
-    if (e != cudaSuccess) return e;
-    attr_set = true;
-  }
+  static int nsm_dev[kMaxDevices] = {};
+  int nsm = 0;
+  cudaError_t e = kernel_setup(nsm_dev, attn_bwd_main_d128_kernel<DH>, C::SMEM_BYTES, &nsm);
+  if (e != cudaSuccess) return e;
   dim3 grid(p.nkt, p.H, p.B);
   attn_bwd_main_d128_kernel<DH><<<grid, C::THREADS, C::SMEM_BYTES, stream>>>(tq, tk, tv, tdo, p);
   return cudaGetLastError();

@@ -478,18 +478,10 @@ template <int DH>
 static cudaError_t launch_persist(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
                                   const CUtensorMap& tdo, const BwdParams& p, cudaStream_t stream) {
   using C = BwdBig<DH>;
-  static bool attr_set = false;
-  static int nsm = 0;
-  if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(attn_bwd_main_d128_persist_kernel<DH>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_BYTES);
-    if (e != cudaSuccess) return e;
-    int dev = 0;
-    if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
-    if ((e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
-    if (nsm < 1) nsm = 1;
-    attr_set = true;
-  }
+  static int nsm_dev[kMaxDevices] = {};
+  int nsm = 0;
+  cudaError_t e = kernel_setup(nsm_dev, attn_bwd_main_d128_persist_kernel<DH>, C::SMEM_BYTES, &nsm);
+  if (e != cudaSuccess) return e;
   // One CTA per SM (shared memory allows no more), stride coprime with the key-tile count:
   // every CTA then sees every key-tile position, whose step counts differ.
   const long long items = (long long)p.nkt * p.H * p.B;

@@ -513,20 +513,13 @@ template <int D>
 static cudaError_t launch_fwd_d(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
                                const FwdParams& p, cudaStream_t stream) {
   using C = FwdCfg<D>;
-  static bool attr_set = false;
-  static int nsm = 0;
-  if (!attr_set) {
-    cudaError_t e =
-        cudaFuncSetAttribute(attn_fwd_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_BYTES);
-    if (e != cudaSuccess) return e;
-    int dev = 0;
-    if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
-    if ((e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
-    if (nsm < 1) nsm = 1;
-    attr_set = true;
-  }
-  // One CTA per SM (shared memory allows no more) walking items; a stride coprime with the
-  // pairs per (sequence, head) gives every CTA every pair position (their key-tile counts differ).
+  static int nsm_dev[kMaxDevices] = {};
+  int nsm = 0;
+  cudaError_t e = kernel_setup(nsm_dev, attn_fwd_kernel<D>, C::SMEM_BYTES, &nsm);
+  if (e != cudaSuccess) return e;
+  // One CTA per SM (shared memory allows no more) walking items: the first G in order, the
+  // rest claimed. G is kept coprime with the pairs per (sequence, head), so the first round
+  // of items mixes pair positions (their key-tile counts differ).
   const int nqp = (p.nqt + 1) / 2;
   const long long items = (long long)nqp * p.H * p.B;
   long long G = items < nsm ? items : nsm;
@@ -539,8 +532,7 @@ static cudaError_t launch_fwd_d(const CUtensorMap& tq, const CUtensorMap& tk, co
     return x;
   };
   while (G > 1 && gcd(G, nqp) != 1) G--;
-  cudaError_t e = cudaMemsetAsync(p.work_ctr, 0, sizeof(unsigned int), stream);  // the claim counter
-  if (e != cudaSuccess) return e;
+  if ((e = cudaMemsetAsync(p.work_ctr, 0, sizeof(unsigned int), stream)) != cudaSuccess) return e;  // the claim counter
   attn_fwd_kernel<D><<<(unsigned)G, C::THREADS, C::SMEM_BYTES, stream>>>(tq, tk, tv, p);
   return cudaGetLastError();
 }

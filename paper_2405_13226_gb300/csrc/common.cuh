@@ -171,6 +171,29 @@ struct RopeParams {
   RopeFreq f;
 };
 
+// One-time setup of a kernel per device: its dynamic shared-memory limit (a function
+// attribute of each device's context, so set on every device the process launches on) and
+// the device's SM count. `nsm` caches the count per device ordinal (0: not set up); a race
+// between host threads only repeats the setup.
+constexpr int kMaxDevices = 64;
+template <typename Kernel>
+inline cudaError_t kernel_setup(int (&nsm)[kMaxDevices], Kernel kernel, int smem_bytes, int* nsm_out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+  if (nsm[dev] == 0) {
+    if (smem_bytes > 0 &&
+        (e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes)) != cudaSuccess)
+      return e;
+    int n = 0;
+    if ((e = cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
+    nsm[dev] = n < 1 ? 1 : n;
+  }
+  *nsm_out = nsm[dev];
+  return cudaSuccess;
+}
+
 // Launchers (defined in attn_fwd.cu / attn_bwd.cu / rope.cu); return a cudaError_t.
 cudaError_t launch_attn_fwd(int d, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
                             const FwdParams& p, cudaStream_t stream);
