@@ -485,6 +485,7 @@ static cudaError_t launch_persist(const CUtensorMap& tq, const CUtensorMap& tk, 
   // One CTA per SM (shared memory allows no more), stride coprime with the key-tile count:
   // every CTA then sees every key-tile position, whose step counts differ.
   const long long items = (long long)p.nkt * p.H * p.B;
+  if (items > 2147483647LL - 4096) return cudaErrorInvalidValue;  // item indices are int
   long long G = items < nsm ? items : nsm;
   auto gcd = [](long long x, long long y) {
     while (y) {

@@ -522,6 +522,7 @@ static cudaError_t launch_fwd_d(const CUtensorMap& tq, const CUtensorMap& tk, co
   // of items mixes pair positions (their key-tile counts differ).
   const int nqp = (p.nqt + 1) / 2;
   const long long items = (long long)nqp * p.H * p.B;
+  if (items > 2147483647LL - 4096) return cudaErrorInvalidValue;  // item indices (and claims past the end) are int
   long long G = items < nsm ? items : nsm;
   auto gcd = [](long long x, long long y) {
     while (y) {
