@@ -144,12 +144,15 @@ dd_status dd_attn_bwd_phases(const dd_attn_desc* desc, const void* q, const void
  * library keeps in device global memory (every GPU that loads the library
  * holds it until the process exits). Sizes whose bwd workspace
  * (dd_attn_workspace_size(desc, 1)) exceeds that return DD_ERR_WORKSPACE with
- * nothing launched. It calls no cudaMalloc / cudaFree. The first call on a
- * device looks up the array's device address (make it before any stream
- * capture). All calls share the array: calls whose kernels overlap on the GPU
- * race, so order them on one stream. device_status (device memory, may be
- * NULL) receives this call's device status word (0, or
- * DD_ERR_DEVICE_TIMEOUT), copied on `stream` after the backward. */
+ * nothing launched; a bad descriptor returns the same code as dd_attn_bwd.
+ * It calls no cudaMalloc / cudaFree. The first call on a device looks up the
+ * array's device address (make it before any stream capture); that address
+ * belongs to the device's context, so do not use this entry point on a device
+ * after cudaDeviceReset in the same process. All calls share the array: calls
+ * whose kernels overlap on the GPU race, so order them on one stream.
+ * device_status (device memory, may be NULL) receives this call's device
+ * status word (0, or DD_ERR_DEVICE_TIMEOUT), copied on `stream` after the
+ * backward. */
 #define DD_NOALLOC_SCRATCH_BYTES ((size_t)32 << 20)
 dd_status dd_attn_bwd_noalloc(const dd_attn_desc* desc, const void* q, const void* k, const void* v,
                               const void* o, const void* dO, const float* lse, void* dq, void* dk, void* dv,

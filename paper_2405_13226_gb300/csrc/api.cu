@@ -1,5 +1,6 @@
 // Host side of the C ABI declared in include/ddattn.h: argument checks,
 // TMA tensor maps, workspace layout, launches and the device status word.
+#include <atomic>
 #include <cmath>
 #include <cstdint>
 #include <cstdlib>
@@ -62,16 +63,18 @@ size_t rope_rows_bytes(const dd_attn_desc* d) {
   return has_rope(d) ? align256((size_t)d->L * (d->d / 2) * sizeof(float2)) : 0;
 }
 
+// The driver's tensor-map encoder, looked up once (a function-local static initialised by
+// its first caller; concurrent first callers wait for that initialisation).
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
-  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-  if (!fn) {
+  static const PFN_cuTensorMapEncodeTiled_v12000 fn = [] {
     void* p = nullptr;
     cudaDriverEntryPointQueryResult q;
     if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
             cudaSuccess &&
         q == cudaDriverEntryPointSuccess)
-      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
-  }
+      return reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    return static_cast<PFN_cuTensorMapEncodeTiled_v12000>(nullptr);
+  }();
   return fn;
 }
 
@@ -92,34 +95,40 @@ bool make_map(CUtensorMap* m, const void* ptr, const dd_attn_desc* d, int box_ro
   return r == CUDA_SUCCESS;
 }
 
+// The current device is an sm_103 part. The verdict is cached per device ordinal
+// (0: not yet checked, 1: supported, 2: not), so host threads driving different GPUs
+// each get their own device's answer.
 dd_status check_device() {
-  static int checked_dev = -1;
-  static dd_status verdict = DD_OK;
+  static std::atomic<int> verdict[kMaxDevices];
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return DD_ERR_CUDA;
-  if (dev != checked_dev) {
+  if (dev < 0 || dev >= kMaxDevices) return DD_ERR_UNSUPPORTED;
+  int v = verdict[dev].load(std::memory_order_acquire);
+  if (v == 0) {
     int major = 0, minor = 0;
     if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
         cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess)
       return DD_ERR_CUDA;
-    verdict = (major == 10 && minor == 3) ? DD_OK : DD_ERR_UNSUPPORTED;
-    checked_dev = dev;
+    v = (major == 10 && minor == 3) ? 1 : 2;
+    verdict[dev].store(v, std::memory_order_release);
   }
-  return verdict;
+  return v == 1 ? DD_OK : DD_ERR_UNSUPPORTED;
 }
 
+// Bound of every device-side wait (DDATTN_WAIT_LIMIT_MS, default 1 s), read once.
 unsigned long long wait_limit_ns() {
-  static unsigned long long v = 0;
-  if (!v) {
+  static const unsigned long long v = [] {
     const char* e = std::getenv("DDATTN_WAIT_LIMIT_MS");
     long long ms = e ? std::atoll(e) : 1000;
     if (ms < 1) ms = 1;
-    v = (unsigned long long)ms * 1000000ull;
-  }
+    return (unsigned long long)ms * 1000000ull;
+  }();
   return v;
 }
 
 }  // namespace
+
+dd_status validate_desc(const dd_attn_desc* desc) { return check_desc(desc); }
 
 // One warp waits on an mbarrier that nothing arrives on; the bounded wait
 // expires after limit_ns and records the timeout in *status.

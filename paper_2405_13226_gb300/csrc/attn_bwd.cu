@@ -540,7 +540,7 @@ template <int D>
 static cudaError_t launch_bwd_d(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
                                 const CUtensorMap& tdo, const BwdParams& p, int phases, cudaStream_t stream) {
   using C = BwdCfg<D>;
-  static int nsm_dev[kMaxDevices] = {};
+  static DeviceCache nsm_dev;
   int nsm = 0;
   // d = 64 has its own main kernel (its shared memory set here); the pre / post kernels use
   // none, and the d = 80 / 128 main kernels are set up by their launchers.

@@ -463,7 +463,7 @@ template <int DH>
 static cudaError_t launch_big(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
                               const CUtensorMap& tdo, const BwdParams& p, cudaStream_t stream) {
   using C = BwdBig<DH>;
-  static int nsm_dev[kMaxDevices] = {};
+  static DeviceCache nsm_dev;
   int nsm = 0;
   cudaError_t e = kernel_setup(nsm_dev, attn_bwd_main_d128_kernel<DH>, C::SMEM_BYTES, &nsm);
   if (e != cudaSuccess) return e;

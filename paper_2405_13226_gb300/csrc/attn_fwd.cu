@@ -513,7 +513,7 @@ template <int D>
 static cudaError_t launch_fwd_d(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
                                const FwdParams& p, cudaStream_t stream) {
   using C = FwdCfg<D>;
-  static int nsm_dev[kMaxDevices] = {};
+  static DeviceCache nsm_dev;
   int nsm = 0;
   cudaError_t e = kernel_setup(nsm_dev, attn_fwd_kernel<D>, C::SMEM_BYTES, &nsm);
   if (e != cudaSuccess) return e;

@@ -1,10 +1,12 @@
 // Shared device/host definitions of the attention kernels.
 #pragma once
+#include <atomic>
 #include <cstdint>
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
+#include "../../include/ddattn.h"
 #include "ptx.cuh"
 
 namespace ddattn {
@@ -173,26 +175,34 @@ struct RopeParams {
 
 // One-time setup of a kernel per device: its dynamic shared-memory limit (a function
 // attribute of each device's context, so set on every device the process launches on) and
-// the device's SM count. `nsm` caches the count per device ordinal (0: not set up); a race
-// between host threads only repeats the setup.
+// the device's SM count. `nsm` caches the count per device ordinal (0: not set up). The
+// entries are atomics: host threads that race on a device's first launch both run the
+// (idempotent) setup and store the same count.
 constexpr int kMaxDevices = 64;
+using DeviceCache = std::atomic<int>[kMaxDevices];
 template <typename Kernel>
-inline cudaError_t kernel_setup(int (&nsm)[kMaxDevices], Kernel kernel, int smem_bytes, int* nsm_out) {
+inline cudaError_t kernel_setup(DeviceCache& nsm, Kernel kernel, int smem_bytes, int* nsm_out) {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
-  if (nsm[dev] == 0) {
+  int have = nsm[dev].load(std::memory_order_acquire);
+  if (have == 0) {
     if (smem_bytes > 0 &&
         (e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes)) != cudaSuccess)
       return e;
     int n = 0;
     if ((e = cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
-    nsm[dev] = n < 1 ? 1 : n;
+    have = n < 1 ? 1 : n;
+    nsm[dev].store(have, std::memory_order_release);
   }
-  *nsm_out = nsm[dev];
+  *nsm_out = have;
   return cudaSuccess;
 }
+
+// Host-side argument check of a descriptor (api.cu): DD_OK, DD_ERR_INVALID_ARG or
+// DD_ERR_UNSUPPORTED, the code every entry point returns for that descriptor.
+dd_status validate_desc(const dd_attn_desc* desc);
 
 // Launchers (defined in attn_fwd.cu / attn_bwd.cu / rope.cu); return a cudaError_t.
 cudaError_t launch_attn_fwd(int d, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,

@@ -15,7 +15,10 @@
 // process exits. Host code cannot use the array's name as a device address:
 // the address is looked up once per device with cudaGetSymbolAddress, with
 // that device current, on the first call made on that device. That first
-// call should therefore come before any stream capture.
+// call should therefore come before any stream capture. The looked-up address
+// belongs to the device's current context: after cudaDeviceReset (which
+// destroys that context and unloads the module) it is stale, so this entry
+// point must not be used on a device that has been reset in this process.
 //
 // All calls share the one array and it keeps the previous call's contents:
 // the status word is cleared at the start of every call and the backward's
@@ -27,6 +30,10 @@
 #include <cuda_runtime.h>
 
 #include "../../include/ddattn.h"
+
+namespace ddattn {
+dd_status validate_desc(const dd_attn_desc* desc);  // api.cu
+}
 
 namespace {
 
@@ -56,9 +63,10 @@ void* scratch_on_current_device() {
 extern "C" dd_status dd_attn_bwd_noalloc(const dd_attn_desc* desc, const void* q, const void* k, const void* v,
                                          const void* o, const void* dO, const float* lse, void* dq, void* dk,
                                          void* dv, int32_t* device_status, void* stream) {
-  const size_t need = dd_attn_workspace_size(desc, 1);
-  if (need == 0) return (desc && desc->d != 64 && desc->d != 128) ? DD_ERR_UNSUPPORTED : DD_ERR_INVALID_ARG;
-  if (need > kNoallocScratchBytes) return DD_ERR_WORKSPACE;
+  // The same code dd_attn_bwd returns for a bad descriptor, then the size limit.
+  const dd_status valid = ddattn::validate_desc(desc);
+  if (valid != DD_OK) return valid;
+  if (dd_attn_workspace_size(desc, 1) > kNoallocScratchBytes) return DD_ERR_WORKSPACE;
   if (!q || !k || !v || !o || !dO || !lse || !dq || !dk || !dv) return DD_ERR_INVALID_ARG;
   void* scratch = scratch_on_current_device();
   if (!scratch) return DD_ERR_CUDA;

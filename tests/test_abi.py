@@ -103,3 +103,27 @@ def test_rope_qk_host_validation(lib):
     assert call(d, p[:3] + [0x40004]) == lib.DD_ERR_INVALID_ARG                   # misaligned k_rot
     assert call(lib.make_desc(2, 256, 2, 96, rope_base=1e4), p) == lib.DD_ERR_UNSUPPORTED
     assert L.dd_rope_qk(None, *p, None) == lib.DD_ERR_INVALID_ARG
+
+
+def test_noalloc_bad_descriptor_codes_match_bwd(lib):
+    """dd_attn_bwd_noalloc returns the code dd_attn_bwd returns for the same bad
+    descriptor, for every supported head dim (d = 80 included), before it looks
+    at the scratch array or any device: nothing is launched."""
+    L = lib.lib()
+    p = [0x10000 * (i + 1) for i in range(9)]
+    for d in (64, 80, 128):
+        bad = []
+        for B, Lq, scale, rope in ((0, 256, None, 0.0), (2, 0, None, 0.0), (2, 256, float("nan"), 0.0),
+                                   (2, 256, None, -1.0)):
+            desc = lib.make_desc(B, Lq, 2, d, scale, None, rope)
+            bad.append(desc)
+        neg_scale = lib.make_desc(2, 256, 2, d)
+        neg_scale.scale = -0.5
+        bad.append(neg_scale)
+        for desc in bad:
+            want = L.dd_attn_bwd(ctypes.byref(desc), *p, 0x100000, 1 << 30, None)
+            got = L.dd_attn_bwd_noalloc(ctypes.byref(desc), *p, None, None)
+            assert want == lib.DD_ERR_INVALID_ARG and got == want, (d, desc.B, desc.L, want, got)
+    unsupported = lib.make_desc(2, 256, 2, 96)
+    assert L.dd_attn_bwd_noalloc(ctypes.byref(unsupported), *p, None, None) == lib.DD_ERR_UNSUPPORTED
+    assert L.dd_attn_bwd_noalloc(None, *p, None, None) == lib.DD_ERR_INVALID_ARG

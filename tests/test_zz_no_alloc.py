@@ -12,7 +12,7 @@ import pytest
 
 from paper_2405_13226_gb300 import workloads as wl
 
-from attn_cases import TOL_GRAD_REL, default_scale, rel_l2, to_device, to_f64
+from attn_cases import TOL_GRAD_REL, default_scale, oracle_full, rel_l2, to_device, to_f64
 
 pytestmark = pytest.mark.gpu
 
@@ -23,20 +23,32 @@ def _noalloc(dd, desc, q, k, v, o, g, lse, dq, dk, dv, status, stream):
                                         status.data_ptr(), ctypes.c_void_p(stream.cuda_stream))
 
 
-@pytest.mark.parametrize("B,L,H,d,doc_mask", [(4, 256, 2, 64, False), (2, 1000, 4, 128, True)])
-def test_noalloc_matches_workspace_entry_point(B, L, H, d, doc_mask):
+# (B, L, H, d, document mask, RoPE base): the d = 64 kernels; the walking d = 128 kernel with
+# documents; d = 80 with RoPE (its (cos, sin) tables live inside the scratch array); the
+# one-CTA-per-key-tile d = 128 kernel (L > 2048).
+CASES = [(4, 256, 2, 64, False, 0.0), (2, 1000, 4, 128, True, 0.0), (2, 640, 2, 80, False, 1e4),
+         (1, 4096, 2, 128, False, 0.0)]
+
+
+@pytest.mark.parametrize("B,L,H,d,doc_mask,rope_base", CASES)
+def test_noalloc_matches_workspace_entry_point(B, L, H, d, doc_mask, rope_base):
+    """Two calls in a row against dd_attn_bwd (same kernels, caller workspace) and
+    against the fp64 oracle, within the parity tolerance."""
     import torch
     from paper_2405_13226_gb300 import ddattn as dd
     scale = default_scale(d)
     qb, kb, vb, gb = wl.attn_inputs(B, L, H, d, seed=11)
     q, k, v, g = (to_device(x) for x in (qb, kb, vb, gb))
-    off = None
+    off, off_np = None, None
     if doc_mask:
         off_np = wl.concat_and_chunk_offsets(4, n_chunks=B, chunk=L)
         off = torch.from_numpy(off_np).cuda()
+    if rope_base:
+        q, k = dd.rope_qk(q, k, rope_base)
     o, lse = dd.fwd(q, k, v, scale, off)
-    ref = dd.bwd(q, k, v, o, g, lse, scale, off)
-    desc = dd.make_desc(B, L, H, d, scale, off)
+    ref = dd.bwd(q, k, v, o, g, lse, scale, off, rope_base=rope_base)
+    _, _, odq, odk, odv = oracle_full(qb, kb, vb, gb, scale, off_np, rope_base)
+    desc = dd.make_desc(B, L, H, d, scale, off, rope_base)
     assert dd.workspace_size(desc, True) <= dd.NOALLOC_SCRATCH_BYTES
     stream = torch.cuda.current_stream()
     for call in range(2):   # the second call reuses the scratch array left by the first
@@ -46,10 +58,12 @@ def test_noalloc_matches_workspace_entry_point(B, L, H, d, doc_mask):
         assert st == dd.DD_OK, dd.status_string(st)
         torch.cuda.synchronize()
         assert int(status.item()) == 0, "device status of call %d" % call
-        for name, got, want in (("dq", dq, ref[0]), ("dk", dk, ref[1]), ("dv", dv, ref[2])):
-            err = rel_l2(to_f64(got), to_f64(want))
-            assert err <= TOL_GRAD_REL, (call, name, err)
+        for name, got, want, orc in (("dq", dq, ref[0], odq), ("dk", dk, ref[1], odk), ("dv", dv, ref[2], odv)):
             assert np.isfinite(to_f64(got)).all(), (call, name)
+            err = rel_l2(to_f64(got), to_f64(want))
+            assert err <= TOL_GRAD_REL, (call, name, "vs dd_attn_bwd", err)
+            err = rel_l2(to_f64(got), orc)
+            assert err <= TOL_GRAD_REL, (call, name, "vs oracle", err)
 
 
 def test_noalloc_rejects_sizes_beyond_scratch():
