@@ -201,3 +201,47 @@ def test_many_short_sequences():
     qb, kb, vb, gb = _inputs(32768, 8, 2, 64, seed=14)
     errs = check_sampled(qb, kb, vb, gb, default_scale(64), [(0, 0), (32767, 1), (12345, 0)], n_rand=2)
     print(errs)
+
+
+def _offsets_unlisted_cuts_and_empty_docs(B, L, seed, per_seq=3):
+    """Document offsets that list NO sequence boundary b*L (0 < b < B): every inner
+    boundary falls inside a document, which the kernels must cut there anyway. The
+    list also repeats values (empty documents): 0 twice at the start, B*L twice at
+    the end, and two inner offsets twice."""
+    rng = np.random.default_rng(seed)
+    cand = np.array([t for t in range(1, B * L) if t % L != 0])
+    inner = np.sort(rng.choice(cand, size=per_seq * B, replace=False))
+    dup = rng.choice(inner, size=2, replace=False)
+    off = np.sort(np.concatenate([[0, 0], inner, dup, [B * L, B * L]])).astype(np.int32)
+    assert not any(b * L in set(off.tolist()) for b in range(1, B))
+    assert (np.diff(off) >= 0).all() and (np.diff(off) == 0).sum() >= 4
+    return off
+
+
+@pytest.mark.parametrize("d", [128, 80, 64])
+@pytest.mark.parametrize("B,L", [(3, 1000), (2, 2500)])
+def test_offsets_omit_sequence_cuts_and_repeat(B, L, d):
+    """cu_doc_offsets that omit the sequence boundaries (documents straddle them) and
+    repeat values (empty documents), every element against the oracle. L = 1000 runs
+    the walking backward (at most 16 key tiles), L = 2500 the one-CTA-per-key-tile
+    backward (d = 80, 128)."""
+    off = _offsets_unlisted_cuts_and_empty_docs(B, L, seed=L + d)
+    errs, _ = check_full(*_inputs(B, L, 2, d, seed=L + d), default_scale(d), off)
+    print(errs)
+
+
+@pytest.mark.parametrize("d", [128, 80])
+def test_offsets_without_inner_entries_equal_causal(d):
+    """Offsets [0, B*L] (one document over the whole flattened batch, no boundary
+    listed) give exactly the plain causal result: sequence boundaries always cut."""
+    import torch
+    B, L = 3, 1000
+    qb, kb, vb, gb = _inputs(B, L, 2, d, seed=21)
+    scale = default_scale(d)
+    plain = run_cuda(qb, kb, vb, gb, scale)
+    one_doc = run_cuda(qb, kb, vb, gb, scale, np.array([0, B * L], dtype=np.int32))
+    for a, b in zip(plain, one_doc):
+        if a.dtype == torch.bfloat16:
+            assert torch.equal(a.view(torch.int16), b.view(torch.int16))
+        else:
+            assert torch.equal(a, b)
