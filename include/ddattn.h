@@ -55,6 +55,8 @@
  * launched. A failed launch returns DD_ERR_CUDA. Every wait inside the
  * kernels is bounded; a wait that expires ends the kernel and records
  * DD_ERR_DEVICE_TIMEOUT in the workspace status word (dd_attn_poll_status).
+ * A backward kernel whose dynamic shared memory does not start 1024-aligned
+ * (never seen on sm_103) records DD_ERR_DEVICE_LAYOUT there and returns.
  * Offsets that break the rules above give undefined values but no
  * out-of-bounds access: every derived index is clamped into the sequence.
  */
@@ -74,7 +76,8 @@ typedef enum {
   DD_ERR_UNSUPPORTED = 2,     /* head dim other than 64, 80 or 128, device not sm_103 */
   DD_ERR_WORKSPACE = 3,       /* workspace missing or smaller than required */
   DD_ERR_CUDA = 4,            /* a CUDA runtime call or launch failed */
-  DD_ERR_DEVICE_TIMEOUT = 5   /* a bounded device-side wait expired */
+  DD_ERR_DEVICE_TIMEOUT = 5,  /* a bounded device-side wait expired */
+  DD_ERR_DEVICE_LAYOUT = 6    /* a kernel found its shared-memory base misaligned and did nothing */
 } dd_status;
 
 typedef struct {
@@ -151,8 +154,8 @@ dd_status dd_attn_bwd_phases(const dd_attn_desc* desc, const void* q, const void
  * after cudaDeviceReset in the same process. All calls share the array: calls
  * whose kernels overlap on the GPU race, so order them on one stream.
  * device_status (device memory, may be NULL) receives this call's device
- * status word (0, or DD_ERR_DEVICE_TIMEOUT), copied on `stream` after the
- * backward. */
+ * status word (0, DD_ERR_DEVICE_TIMEOUT or DD_ERR_DEVICE_LAYOUT), copied on
+ * `stream` after the backward. */
 #define DD_NOALLOC_SCRATCH_BYTES ((size_t)32 << 20)
 dd_status dd_attn_bwd_noalloc(const dd_attn_desc* desc, const void* q, const void* k, const void* v,
                               const void* o, const void* dO, const float* lse, void* dq, void* dk, void* dv,

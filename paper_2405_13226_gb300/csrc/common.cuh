@@ -16,6 +16,7 @@ constexpr float kLn2 = 0.6931471805599453f;
 
 // Device status codes (mirror dd_status in include/ddattn.h).
 constexpr int kStatusTimeout = 5;
+constexpr int kStatusLayout = 6;
 
 // Document start of token t (flattened index), per the document-mask rule:
 // the largest offset <= t, never before the start of t's sequence

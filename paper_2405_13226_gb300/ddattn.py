@@ -16,7 +16,8 @@ import torch
 _PKG = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_PKG, "libddattn.so")
 
-DD_OK, DD_ERR_INVALID_ARG, DD_ERR_UNSUPPORTED, DD_ERR_WORKSPACE, DD_ERR_CUDA, DD_ERR_DEVICE_TIMEOUT = range(6)
+(DD_OK, DD_ERR_INVALID_ARG, DD_ERR_UNSUPPORTED, DD_ERR_WORKSPACE, DD_ERR_CUDA, DD_ERR_DEVICE_TIMEOUT,
+ DD_ERR_DEVICE_LAYOUT) = range(7)
 
 
 class DDAttnError(RuntimeError):
