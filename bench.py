@@ -338,8 +338,10 @@ def run_ours(args):
     peak = peaks["bf16_tflops_sustained"]
     roofline = {"kernel": "attn_bwd_main (d=128: walking kernel for L <= 2048, per-key-tile kernel above)", "bound": "tensor", "achieved": main_ach, "peak": peak,
                 "unit": "TFLOP/s", "frac": main_ach / peak, "traffic": measured_traffic(),
-                "traffic_note": "mean dram__bytes_read+write per launch over the six buckets (ncu, "
-                                "profiles/attn_main_kernels_sweep_traffic.md); null if the kernel changed since",
+                "traffic_note": "not measured in this run: mean dram__bytes_read+write per launch over the six "
+                                "buckets, read from the committed ncu summary "
+                                "profiles/attn_main_kernels_sweep_traffic.md (one kernel and one launch per "
+                                "capture), keyed by a hash of the kernel sources; null if they changed since",
                 "peak_kind": "bf16_tflops_sustained (%s)" % peak_src,
                 "share_of_step": main_t / total_ms,
                 "fwd_kernel_tflops": sum(bk.flops_fwd for bk in buckets) * args.steps / (fwd_t * 1e-3) / 1e12,
@@ -367,8 +369,10 @@ def run_ours(args):
         "roofline": roofline,
         "cpu_baseline": cpu,
         "e2e": e2e,
-        # per bucket call: forward, backward pre / main / post (+ RoPE rotation and table)
-        "gpu_launches": args.steps * nb * (4 + (2 if args.rope_base else 0)),
+        # per bucket call: forward, backward pre / main / post (+ RoPE rotation and table);
+        # for L <= 256 the backward main kernel writes dq itself and post launches nothing
+        "gpu_launches": args.steps * sum(bwd_launches(bk.L, D) + 1 + (2 if args.rope_base else 0)
+                                         for bk in buckets),
         "clocks": clk.summary(),
     }
     line.update(extras)
@@ -377,6 +381,12 @@ def run_ours(args):
     if world > 1:
         import torch.distributed as dist
         dist.destroy_process_group()
+
+
+def bwd_launches(L: int, d: int) -> int:
+    """Kernels one backward call launches: pre, main and post, except that for sequences of
+    at most two 128-key tiles at d = 80 / 128 the main kernel writes dq itself (no post)."""
+    return 2 if d != 64 and (L + 127) // 128 <= 2 else 3
 
 
 def dm_pair_fractions(n_seeds: int) -> np.ndarray:

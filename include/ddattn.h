@@ -130,7 +130,10 @@ dd_status dd_attn_bwd(const dd_attn_desc* desc, const void* q, const void* k, co
  * DD_BWD_MAIN (P recompute and the five contractions; dK, dV and the fp32 dQ
  * accumulator), DD_BWD_POST (dq = bf16(scale * accumulator)). With RoPE the
  * PRE phase also fills the (cos, sin) table, and MAIN / POST rotate dk / dq
- * back with it. `phases` is a
+ * back with it. For sequences of at most 256 tokens at d = 80 / 128, MAIN
+ * writes dq itself (its CTAs own whole (sequence, head) pairs and keep their
+ * fp32 dQ rows in the accumulator, one region per CTA), PRE does not zero the
+ * accumulator and POST launches nothing. `phases` is a
  * bit mask; issuing the phases in this order, with the same arguments and
  * workspace, equals one dd_attn_bwd call (dd_attn_bwd = all three). */
 enum { DD_BWD_PRE = 1, DD_BWD_MAIN = 2, DD_BWD_POST = 4, DD_BWD_ALL = 7 };

@@ -256,6 +256,7 @@ dd_status dd_attn_bwd_phases(const dd_attn_desc* desc, const void* q, const void
   p.rope_tab = has_rope(desc) ? reinterpret_cast<float4*>(rope_base) : nullptr;
   p.rope_tab_rows = has_rope(desc) ? reinterpret_cast<float2*>(rope_base + rope_tab_bytes(desc)) : nullptr;
   p.rope = has_rope(desc) ? rope_freq(desc) : RopeFreq{};
+  p.dq_owned = 0;  // chosen by the launcher from the key-tile count
   p.status = static_cast<int*>(ws);
   p.timeout_ns = wait_limit_ns();
   cudaError_t e = launch_attn_bwd(desc->d, tq, tk, tv, tdo, p, phases, static_cast<cudaStream_t>(stream));

@@ -112,7 +112,7 @@ __global__ void __launch_bounds__(256) attn_bwd_pre_kernel(const BwdParams p) {
         g[u] = make_uint4(0u, 0u, 0u, 0u);
       }
     }
-    {  // zero the accumulator span of these rows (flat), interleaving writes with the reads
+    if (!p.dq_owned) {  // zero the accumulator span of these rows (flat), interleaving writes with the reads
       constexpr int AC = acc_cols<D>();
       float4* acc4 = reinterpret_cast<float4*>(p.dq_acc) + r0 * (AC / 4);
       const long long lim = (nrows - r0 < RPW * U ? nrows - r0 : RPW * U) * (AC / 4);
@@ -165,6 +165,7 @@ __global__ void __launch_bounds__(256) attn_bwd_pre_kernel(const BwdParams p) {
     }
   }
   // zero the rest of the dQ accumulator (past nrows * acc_cols: the padded rows)
+  if (p.dq_owned) return;  // the main kernel's first partial of every query tile is a store
   const long long n4 = (long long)p.B * p.H * p.L128 * acc_cols<D>() / 4;
   float4* acc4 = reinterpret_cast<float4*>(p.dq_acc);
   for (long long t = nrows * (acc_cols<D>() / 4) + tid; t < n4; t += stride) acc4[t] = make_float4(0.f, 0.f, 0.f, 0.f);
@@ -536,10 +537,23 @@ __global__ void __launch_bounds__(320, 1)
   }
 }
 
+// Sequences of at most this many key tiles take the dQ-owned walk of the d = 80 / 128 main
+// kernel: its CTAs own whole (sequence, head) pairs, keep their fp32 dQ rows in an L2-resident
+// slot and write bf16 dq themselves, so the accumulator is neither zeroed (pre) nor converted
+// (post). Measured against the shared accumulator in one process (H = 16, d = 128, 65536
+// tokens): backward 0.742 -> 0.709 ms at L = 256, but 0.912 -> 0.943 at 512, 1.178 -> 1.423
+// at 1024 and 1.642 -> 1.929 at 2048. Per CTA the slot and the re-read window of its pair's
+// Q / dO tiles grow with L (0.5 MB each at L = 1024, times 152 CTAs), so they fall out of L2,
+// while the per-key-tile walk shares each Q / dO tile between the CTAs that work on one pair
+// at the same time; and each pair's conversion holds the drain warps.
+constexpr int kDqOwnedMaxTiles = 2;
+
 template <int D>
 static cudaError_t launch_bwd_d(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
-                                const CUtensorMap& tdo, const BwdParams& p, int phases, cudaStream_t stream) {
+                                const CUtensorMap& tdo, const BwdParams& p_in, int phases, cudaStream_t stream) {
   using C = BwdCfg<D>;
+  BwdParams p = p_in;
+  p.dq_owned = (D != 64 && p.nkt <= kDqOwnedMaxTiles) ? 1 : 0;
   static DeviceCache nsm_dev;
   int nsm = 0;
   // d = 64 has its own main kernel (its shared memory set here); the pre / post kernels use
@@ -567,7 +581,7 @@ static cudaError_t launch_bwd_d(const CUtensorMap& tq, const CUtensorMap& tk, co
       if ((e = cudaGetLastError()) != cudaSuccess) return e;
     }
   }
-  if (phases & 4) {
+  if ((phases & 4) && !p.dq_owned) {
     attn_bwd_post_kernel<D><<<ew_blocks, 256, 0, stream>>>(p);
     e = cudaGetLastError();
   }

@@ -20,7 +20,41 @@
 
 namespace ddattn {
 
-template <int DH>
+// dq rows [r0, r0 + 128) of one (sequence, head), columns 32 w .. 32 w + NV - 1 (NV = 32, or
+// 16 for the last chunk at d = 80), from the fp32 slot rows acc_w (chunk w, row-major
+// [L128][32]): dq = bf16(scale * acc), rotated back (R^T) with RoPE. Lane l converts rows
+// r0 + l, r0 + l + 32, ...; a row is 4 NV contiguous bytes of the slot and 2 NV of dq.
+template <int D, int NV>
+__device__ __forceinline__ void dq_owned_convert(const BwdParams& p, const float* acc_w, long long seq0, int h,
+                                                 int r0, int w, int lane) {
+#pragma unroll 1
+  for (int rr = lane; rr < 128; rr += 32) {
+    const int row = r0 + rr;
+    if (row >= p.L) break;
+    const float4* src = reinterpret_cast<const float4*>(acc_w + (long long)row * 32);
+    float f[32];
+#pragma unroll
+    for (int q = 0; q < NV / 4; q++) {
+      const float4 x = src[q];
+      f[4 * q] = x.x * p.scale;
+      f[4 * q + 1] = x.y * p.scale;
+      f[4 * q + 2] = x.z * p.scale;
+      f[4 * q + 3] = x.w * p.scale;
+    }
+    if (p.rope_tab_rows) {  // pairs j = 16 w + u at position row
+      const float4* cs = reinterpret_cast<const float4*>(p.rope_tab_rows + (long long)row * (D / 2) + w * 16);
+#pragma unroll
+      for (int u = 0; u < NV / 4; u++) {
+        const float4 c = cs[u];
+        rope_unrotate_pair(f[4 * u], f[4 * u + 1], c.x, c.y);
+        rope_unrotate_pair(f[4 * u + 2], f[4 * u + 3], c.z, c.w);
+      }
+    }
+    store_row(p.dq + ((seq0 + row) * p.H + h) * D + w * 32, f, NV);
+  }
+}
+
+template <int DH, int WALK>
 __global__ void __launch_bounds__(512, 1)
     attn_bwd_main_d128_persist_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                                       const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmDO,
@@ -34,9 +68,8 @@ __global__ void __launch_bounds__(512, 1)
   Bwd128Bars* bars = reinterpret_cast<Bwd128Bars*>(smem + C::OFF_BAR);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
-  // CTA c works on items c, c + G, c + 2G ... (G = gridDim.x); per-step barrier phases and
+  // CTA c works on the items of bwd_walk_item (G = gridDim.x); per-step barrier phases and
   // TMEM region roles follow the CTA's running step count g across items.
-  const int n_items = p.nkt * p.H * p.B;
   Watchdog wd{&bars->abort_flag, p.status, p.timeout_ns};
 
   if (threadIdx.x == 0) {
@@ -89,7 +122,7 @@ __global__ void __launch_bounds__(512, 1)
       prefetch_tmap(&tmDO);
       int q_issued = 0, kv_issued = 0, g0 = 0, ic = 0;
       bool ok = true;
-      for (int it = blockIdx.x; ok && it < n_items; it += gridDim.x, ic++) {
+      for (int it; ok && (it = bwd_walk_item<WALK>(p, ic)) >= 0; ic++) {
         const BwdItem I = bwd_item<C::BN, BQ>(p, it);
         for (int i = 0; i < I.nq; i++) {
           const int g = g0 + i, s = g & 1;
@@ -139,7 +172,7 @@ __global__ void __launch_bounds__(512, 1)
       const uint64_t dO_mn0 = sdesc_sw128(smem_u32(sDO), C::BLK, 1024);
       bool ok = true;
       int g0 = 0, ic = 0;
-      for (int it = blockIdx.x; ok && it < n_items; it += gridDim.x, ic++) {
+      for (int it; ok && (it = bwd_walk_item<WALK>(p, ic)) >= 0; ic++) {
         const int nq = bwd_item<C::BN, BQ>(p, it).nq;
         // The item's first S^T and dP^T, into R[g0 % 2] (the previous step's dP^T region,
         // once the P / dS warps have read it) and R[(g0 + 1) % 2] (its dQ^T region, once drained).
@@ -264,7 +297,7 @@ __global__ void __launch_bounds__(512, 1)
     const float sl2 = p.scale_log2;
     bool ok = true;
     int g0 = 0, ic = 0;
-    for (int it = blockIdx.x; ok && it < n_items; it += gridDim.x, ic++) {
+    for (int it; ok && (it = bwd_walk_item<WALK>(p, ic)) >= 0; ic++) {
     const BwdItem I = bwd_item<C::BN, BQ>(p, it);
     const int h = I.h, m_lo = I.m_lo, nq = I.nq;
     const long long seq0 = I.seq0;
@@ -407,11 +440,15 @@ __global__ void __launch_bounds__(512, 1)
     const bool drains = w < C::NCH;               // d = 80: the fourth chunk (rows 96..127 of dQ^T) is zero
     bool ok = true;
     int g0 = 0, ic = 0;
-    for (int it = blockIdx.x; ok && it < n_items; it += gridDim.x, ic++) {
+    for (int it; ok && (it = bwd_walk_item<WALK>(p, ic)) >= 0; ic++) {
     const BwdItem I = bwd_item<C::BN, BQ>(p, it);
     const int h = I.h, m_lo = I.m_lo, nq = I.nq, kv0 = I.kv0;
     const long long seq0 = I.seq0;
-    float* acc_w = p.dq_acc + (I.vec0 * C::NCH + (long long)w * p.L128) * 32;  // chunk w of this (b, h)
+    // Chunk w of the fp32 dQ rows: the (b, h) region of the shared accumulator, or, with dQ
+    // owned, this CTA's own slot (the region of index blockIdx.x, reused for every pair the
+    // CTA owns, so it stays in L2).
+    float* acc_w = WALK == kWalkOwned ? p.dq_acc + ((long long)blockIdx.x * C::NCH + w) * p.L128 * 32
+                                      : p.dq_acc + (I.vec0 * C::NCH + (long long)w * p.L128) * 32;
     for (int i = 0; i < nq; i++) {
       const int g = g0 + i;
       ok = __all_sync(0xffffffffu, mbar_wait(&bars->dq_full, g & 1, wd));
@@ -439,7 +476,15 @@ __global__ void __launch_bounds__(512, 1)
         fence_proxy_async_smem();
         __syncwarp();
         if (lane == 0) {
-          bulk_reduce_add_f32(acc_w + (long long)(q0 + 32 * c) * 32, stg, 32 * 32 * 4);
+          float* dst = acc_w + (long long)(q0 + 32 * c) * 32;
+          if (WALK == kWalkOwned && i == 0) {
+            bulk_store(dst, stg, 32 * 32 * 4);  // the query tile's first partial
+          } else {
+            // With dQ owned, this block's first partial (a store) is at least 8 groups back:
+            // 3 - c after it in its step, 4 in the next item's diagonal step, c before this one.
+            if (WALK == kWalkOwned) bulk_wait<7>();
+            bulk_reduce_add_f32(dst, stg, 32 * 32 * 4);
+          }
           bulk_commit();
         }
       }
@@ -463,6 +508,25 @@ __global__ void __launch_bounds__(512, 1)
       tc_fence_before();
       mbar_arrive(&bars->dk_free);  // dK of this item has left TMEM
     }
+    // dQ owned: the query tiles whose last contributor is this key tile are complete once
+    // this warp's copies have landed; convert its chunk of their rows to bf16 dq.
+    if (WALK == kWalkOwned && ok && drains) {
+      uint32_t done = 0;  // bit i: query tile m_lo + i (nq <= 16)
+      for (int i = 0; i < nq; i++)
+        if (bwd_last_contributor(p, seq0, m_lo + i) == I.n) done |= 1u << i;
+      if (done) {
+        if (lane == 0) bulk_wait<0>();
+        __syncwarp();
+        fence_proxy_async_global();
+        for (int i = 0; i < nq; i++) {
+          if (!(done & (1u << i))) continue;
+          if (D - 32 * w >= 32) dq_owned_convert<D, 32>(p, acc_w, seq0, h, (m_lo + i) * BQ, w, lane);
+          else dq_owned_convert<D, 16>(p, acc_w, seq0, h, (m_lo + i) * BQ, w, lane);
+        }
+        __syncwarp();
+        fence_proxy_async_global();  // these reads before the next pair's copies into the slot
+      }
+    }
     g0 += nq;
     }
     if (lane == 0) bulk_wait<0>();  // every reduction of this CTA has landed
@@ -478,30 +542,43 @@ __global__ void __launch_bounds__(512, 1)
   }
 }
 
-template <int DH>
-static cudaError_t launch_persist(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
-                                  const CUtensorMap& tdo, const BwdParams& p, cudaStream_t stream) {
+template <int DH, int WALK>
+static cudaError_t launch_walk(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
+                               const CUtensorMap& tdo, const BwdParams& p, cudaStream_t stream) {
   using C = BwdBig<DH>;
   static DeviceCache nsm_dev;
   int nsm = 0;
-  cudaError_t e = kernel_setup(nsm_dev, attn_bwd_main_d128_persist_kernel<DH>, C::SMEM_BYTES, &nsm);
+  cudaError_t e = kernel_setup(nsm_dev, attn_bwd_main_d128_persist_kernel<DH, WALK>, C::SMEM_BYTES, &nsm);
   if (e != cudaSuccess) return e;
-  // One CTA per SM (shared memory allows no more), stride coprime with the key-tile count:
-  // every CTA then sees every key-tile position, whose step counts differ.
   const long long items = (long long)p.nkt * p.H * p.B;
   if (items > 2147483647LL - 4096) return cudaErrorInvalidValue;  // item indices are int
-  long long G = items < nsm ? items : nsm;
-  auto gcd = [](long long x, long long y) {
-    while (y) {
-      const long long t = x % y;
-      x = y;
-      y = t;
-    }
-    return x;
-  };
-  while (G > 1 && gcd(G, p.nkt) != 1) G--;
-  attn_bwd_main_d128_persist_kernel<DH><<<(unsigned)G, C::THREADS, C::SMEM_BYTES, stream>>>(tq, tk, tv, tdo, p);
+  long long G = items < nsm ? items : nsm;  // one CTA per SM (shared memory allows no more)
+  if (WALK == kWalkOwned) {
+    // over the (sequence, head) pairs; CTA c uses slot c
+    const long long pairs = (long long)p.B * p.H;
+    G = pairs < nsm ? pairs : nsm;
+  } else {
+    // stride coprime with the key-tile count: every CTA then sees every key-tile position,
+    // whose step counts differ
+    auto gcd = [](long long x, long long y) {
+      while (y) {
+        const long long t = x % y;
+        x = y;
+        y = t;
+      }
+      return x;
+    };
+    while (G > 1 && gcd(G, p.nkt) != 1) G--;
+  }
+  attn_bwd_main_d128_persist_kernel<DH, WALK><<<(unsigned)G, C::THREADS, C::SMEM_BYTES, stream>>>(tq, tk, tv, tdo, p);
   return cudaGetLastError();
+}
+
+template <int DH>
+static cudaError_t launch_persist(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
+                                  const CUtensorMap& tdo, const BwdParams& p, cudaStream_t stream) {
+  if (p.dq_owned) return launch_walk<DH, kWalkOwned>(tq, tk, tv, tdo, p, stream);
+  return launch_walk<DH, kWalkStatic>(tq, tk, tv, tdo, p, stream);
 }
 
 cudaError_t launch_attn_bwd_main_d128_persist(int d, const CUtensorMap& tq, const CUtensorMap& tk,

@@ -80,4 +80,35 @@ __device__ __forceinline__ BwdItem bwd_item(const BwdParams& p, int it) {
   return I;
 }
 
+// How the CTAs of the walking backward kernel get their items (a template parameter, so
+// that each kernel instance holds only its own walk's code).
+enum BwdWalk { kWalkStatic = 0, kWalkOwned = 1 };
+
+// The w-th item of this CTA's walk (w = 0, 1, ...), or -1 past its end. Two orders:
+//   * per key tile: items c, c + G, c + 2G, ... (c = blockIdx.x, G = gridDim.x coprime with
+//     the key-tile count), so the CTAs share the (sequence, head) pairs' dQ rows and reduce
+//     their partials into one fp32 accumulator that the post kernel converts;
+//   * dQ owned (kWalkOwned): CTA c owns the (sequence, head) pairs c, c + G, ... and walks
+//     each one's key tiles from the last to the first. All partials of a query tile then
+//     come from one CTA, the first of them from the key tile on its diagonal (step 0 of that
+//     item: no key tile after it reaches back to the tile, and every earlier one reaches it
+//     only after), and the last from the key tile that holds the document start of the
+//     tile's first row.
+template <int WALK>
+__device__ __forceinline__ int bwd_walk_item(const BwdParams& p, int w) {
+  if (WALK != kWalkOwned) {
+    const long long it = blockIdx.x + (long long)w * gridDim.x;
+    return it < (long long)p.nkt * p.H * p.B ? (int)it : -1;
+  }
+  const long long bh = blockIdx.x + (long long)(w / p.nkt) * gridDim.x;
+  if (bh >= (long long)p.B * p.H) return -1;
+  return (int)(bh * p.nkt + (p.nkt - 1 - w % p.nkt));
+}
+
+// Key tile (relative to the sequence) of the last dQ contributor of query tile qt in the
+// dQ-owned walk: the tile holding the document start of the query tile's first row.
+__device__ __forceinline__ int bwd_last_contributor(const BwdParams& p, long long seq0, int qt) {
+  return (int)((doc_start(p.offsets, p.n_offsets, seq0 + (long long)qt * 128, seq0) - seq0) / 128);
+}
+
 }  // namespace ddattn

@@ -158,8 +158,9 @@ struct BwdParams {
   __nv_bfloat16* dk;
   __nv_bfloat16* dv;
   float4* rope_tab;       // (cos, sin) of m theta_j (layout of rope_tab_index), or nullptr without RoPE
-  float2* rope_tab_rows;  // the same values row-major [L, d/2] (read by the dq post kernel)
+  float2* rope_tab_rows;  // the same values row-major [L, d/2] (read where dq is written)
   RopeFreq rope;     // frequencies that fill rope_tab
+  int dq_owned;      // the main kernel's CTAs own whole (sequence, head) pairs and write dq themselves
   int* status;
   unsigned long long timeout_ns;
 };

@@ -159,6 +159,20 @@ __device__ __forceinline__ void bulk_reduce_add_f32(float* gdst, const void* ssr
                : "memory");
 }
 
+// Plain bulk copy of `bytes` of shared memory to global memory (both 16-byte
+// aligned, bytes a multiple of 16), bulk-group completion.
+__device__ __forceinline__ void bulk_store(void* gdst, const void* ssrc, uint32_t bytes) {
+  asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(reinterpret_cast<uint64_t>(gdst)),
+               "r"(smem_u32(ssrc)), "r"(bytes)
+               : "memory");
+}
+
+// Order this thread's async-proxy global accesses (completed bulk copies and
+// reductions) with its later generic-proxy accesses of the same memory.
+__device__ __forceinline__ void fence_proxy_async_global() {
+  asm volatile("fence.proxy.async.global;" ::: "memory");
+}
+
 // Warpgroup register reallocation: every warp of the warpgroup executes it;
 // the increases must fit in what the decreases and the launch leave free.
 template <uint32_t N>

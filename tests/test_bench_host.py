@@ -36,3 +36,12 @@ def test_smi_index_follows_visible_devices(monkeypatch):
     assert bench.smi_index(0) == "3" and bench.smi_index(1) == "GPU-abc"
     monkeypatch.delenv("CUDA_VISIBLE_DEVICES")
     assert bench.smi_index(2) == "2"
+
+
+def test_backward_launch_count():
+    """Pre, main and post per backward call, except for sequences of at most two key tiles
+    at d = 80 / 128, whose main kernel writes dq (no post launch); d = 64 always has three."""
+    import bench
+    assert bench.bwd_launches(256, 128) == 2 and bench.bwd_launches(130, 80) == 2
+    assert bench.bwd_launches(257, 128) == 3 and bench.bwd_launches(8192, 128) == 3
+    assert bench.bwd_launches(256, 64) == 3
