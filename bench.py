@@ -228,7 +228,8 @@ class Bucket:
         shape = (B, L, Hh, Dh)
         self.q, self.k, self.v, self.g = (x.view(shape) for x in (q, k, v, g))
         if rope_base:
-            # the attention reads the rotated q, k (written by rope_qk each step)
+            # the attention reads the rotated q, k, written each step by the forward
+            # (dd_attn_fwd_rope) or, in the separate form, by rope_qk
             self.q_raw, self.k_raw = self.q, self.k
             self.q, self.k = (x.view(shape) for x in qk_rot)
         self.o = torch.empty_like(self.q)
@@ -246,7 +247,14 @@ class Bucket:
 
     def fwd(self, stream):
         if self.rope_base:
-            self.rope(stream)
+            self.dd.fwd_rope(self.q_raw, self.k_raw, self.v, self.rope_base, None, self.off, self.o, self.lse, self.q,
+                             self.k, self.ws, stream)
+        else:
+            self.dd.fwd(self.q, self.k, self.v, None, self.off, self.o, self.lse, self.ws, stream)
+
+    def fwd_separate(self, stream):
+        """RoPE as its own pass (rope_qk), then the plain forward on the rotated q, k."""
+        self.rope(stream)
         self.dd.fwd(self.q, self.k, self.v, None, self.off, self.o, self.lse, self.ws, stream)
 
     def bwd(self, stream, phases=None):
@@ -369,9 +377,11 @@ def run_ours(args):
         "roofline": roofline,
         "cpu_baseline": cpu,
         "e2e": e2e,
-        # per bucket call: forward, backward pre / main / post (+ RoPE rotation and table);
-        # for L <= 256 the backward main kernel writes dq itself and post launches nothing
-        "gpu_launches": args.steps * sum(bwd_launches(bk.L, D) + 1 + (2 if args.rope_base else 0)
+        # per bucket call: forward, backward pre / main / post; with RoPE the forward's and the
+        # backward's (cos, sin) table fills and, above 512 tokens, the forward's k pass. For
+        # L <= 256 the backward main kernel writes dq itself and post launches nothing.
+        "gpu_launches": args.steps * sum(bwd_launches(bk.L, D) + 1
+                                         + ((2 + (1 if bk.L > 512 else 0)) if args.rope_base else 0)
                                          for bk in buckets),
         "clocks": clk.summary(),
     }
@@ -519,28 +529,38 @@ def extra_workloads(ddattn, q, k, v, g, buckets, ws, stream, peaks, dev):
     out["pack8k_dm"] = {"workload": "8 best-fit-decreasing bins x 8192, H=16, d=128, document-masked, seeds 0..3; "
                                     "10 timed calls after 3 warm-up calls per seed",
                         "ms_per_step_mean": float(np.mean([x["ms"] for x in pk])), "per_seed": pk}
-    # RoPE (f_b = 100k) on the bucket sweep: rotation kernel + forward + backward
-    # with R^T fused into the dq / dk outputs, against the same step without RoPE
+    # RoPE (f_b = 100k) on the bucket sweep: the forward that rotates q, k itself
+    # (dd_attn_fwd_rope) + backward with R^T fused into the dq / dk outputs, against the
+    # same step without RoPE and against the separate rotation pass (rope_qk + fwd + bwd)
     qr, kr = torch.empty_like(q), torch.empty_like(k)
     rdesc = [ddattn.make_desc(T // L, L, H, D, None, None, 1e5) for L in wl.BUCKETS]
     rws = ddattn.new_workspace(max(rdesc, key=lambda x: ddattn.workspace_size(x)), dev)
     rope_rows = []
     for bk0 in buckets:
         bk = Bucket(ddattn, q, k, v, g, bk0.B, bk0.L, H, ws=rws, rope_base=1e5, qk_rot=(qr, kr))
-        ms = time_calls(lambda: (bk.fwd(stream), bk.bwd(stream)), 3, 1, stream)
-        ms_plain = time_calls(lambda: (bk0.fwd(stream), bk0.bwd(stream)), 3, 1, stream)
+        ms = time_calls(lambda: (bk.fwd(stream), bk.bwd(stream)), 5, 2, stream)
+        ms_sep = time_calls(lambda: (bk.fwd_separate(stream), bk.bwd(stream)), 5, 2, stream)
+        ms_plain = time_calls(lambda: (bk0.fwd(stream), bk0.bwd(stream)), 5, 2, stream)
+        fwd_ms = time_calls(lambda: bk.fwd(stream), 10, 2, stream)
+        fwd_sep_ms = time_calls(lambda: bk.fwd_separate(stream), 10, 2, stream)
         rope_ms = time_calls(lambda: bk.rope(stream), 10, 2, stream)
-        rope_rows.append({"L": bk.L, "ms": ms, "ms_without_rope": ms_plain, "rope_kernel_ms": rope_ms,
+        rope_rows.append({"L": bk.L, "ms": ms, "ms_separate_pass": ms_sep, "ms_without_rope": ms_plain,
+                          "fwd_ms": fwd_ms, "fwd_separate_pass_ms": fwd_sep_ms, "rope_kernel_ms": rope_ms,
                           "rope_kernel_GBps": 4 * T * H * D * 2 / (rope_ms * 1e-3) / 1e9,
                           "tflops": bk.flops / (ms * 1e-3) / 1e12})
     st = ddattn.poll_status(rws)
     if st != 0:
         raise RuntimeError("device status %d (%s)" % (st, ddattn.status_string(st)))
     step_rope = sum(x["ms"] for x in rope_rows)
+    step_sep = sum(x["ms_separate_pass"] for x in rope_rows)
     step_plain = sum(x["ms_without_rope"] for x in rope_rows)
-    out["rope_sweep"] = {"workload": "bucket sweep with RoPE f_b=100k: dd_rope_qk + fwd + bwd per bucket",
-                         "ms_per_step": step_rope, "ms_per_step_without_rope": step_plain,
+    out["rope_sweep"] = {"workload": "bucket sweep with RoPE f_b=100k: dd_attn_fwd_rope (rotation in the forward "
+                                     "kernel; k by a pass first above 512 tokens) + bwd per bucket; the separate "
+                                     "form: dd_rope_qk + fwd + bwd",
+                         "ms_per_step": step_rope, "ms_per_step_separate_pass": step_sep,
+                         "ms_per_step_without_rope": step_plain,
                          "overhead": step_rope / step_plain - 1.0,
+                         "overhead_separate_pass": step_sep / step_plain - 1.0,
                          "rope_kernel_frac_of_measured_hbm": float(np.median([x["rope_kernel_GBps"] for x in rope_rows]))
                          / peaks["hbm_gbs"],
                          "per_bucket": rope_rows}

@@ -25,8 +25,10 @@
  *     theta_j = f_b^(-2j/d),
  *     (x_2j, x_2j+1) -> (x_2j cos m theta_j - x_2j+1 sin m theta_j,
  *                        x_2j sin m theta_j + x_2j+1 cos m theta_j).
- *   dd_rope_qk applies it (bf16 out). With desc->rope_base = f_b > 0, the
- *   q and k given to dd_attn_fwd / dd_attn_bwd are the ROTATED ones, and
+ *   dd_attn_fwd_rope applies it inside the forward kernel and also returns the
+ *   rotated q and k; dd_rope_qk applies it as a separate pass (bf16 out). With
+ *   desc->rope_base = f_b > 0, the q and k given to dd_attn_fwd / dd_attn_bwd
+ *   are the ROTATED ones, and
  *   dd_attn_bwd returns dq, dk with respect to the UN-rotated q and k (it
  *   applies the transposed rotation to the rotated-space gradients inside its
  *   kernels). rope_base = 0 means no rotation.
@@ -91,8 +93,9 @@ typedef struct {
   float rope_base;                 /* RoPE base frequency f_b; 0 = no RoPE; else finite and > 0 */
 } dd_attn_desc;
 
-/* Workspace bytes for dd_attn_fwd (for_bwd = 0) or dd_attn_bwd (for_bwd = 1):
- * the status word, and for bwd the fp32 dQ accumulator (B*H*L128*d' floats,
+/* Workspace bytes for dd_attn_fwd / dd_attn_fwd_rope (for_bwd = 0) or
+ * dd_attn_bwd (for_bwd = 1): the status word, for fwd with rope_base > 0 the
+ * fp32 (cos, sin) table [L, d/2] of dd_attn_fwd_rope, and for bwd the fp32 dQ accumulator (B*H*L128*d' floats,
  * d' = 64 for d = 64, else d rounded up to a multiple of 32) plus
  * the per-row D_i and LSE_i*log2(e) vectors [B, H, L128], L128 = L rounded up
  * to a multiple of 128, plus, when rope_base > 0, two copies of the
@@ -116,6 +119,27 @@ dd_status dd_attn_fwd(const dd_attn_desc* desc, const void* q, const void* k, co
  * k_rot == k) is allowed. One bandwidth-bound kernel, no workspace. */
 dd_status dd_rope_qk(const dd_attn_desc* desc, const void* q, const void* k, void* q_rot, void* k_rot,
                      void* stream);
+
+/* Forward with the RoPE rotation fused into the kernel (the rotation above;
+ * Sec. 3 training setup, RoPE base f_b of the f_b ablation table and Table 2):
+ * q and k are the UN-rotated projections. Each 128-row Q tile is loaded once
+ * per forward; the kernel rotates it in shared memory right after its TMA copy
+ * lands and before the tensor core reads it, and writes it to q_rot. For
+ * sequences of at most 4 key tiles (L <= 512) it does the same with every K
+ * tile it loads, and each K tile reaches k_rot from the work item on whose
+ * diagonal it lies. Longer sequences load each K tile in many work items, so
+ * their k is rotated once, into k_rot, by a bandwidth-bound pass on `stream`
+ * before the kernel, which then reads k_rot. The arithmetic is dd_rope_qk's
+ * (fp32, bf16 rounding); the kernel steps the (cos, sin) of a row from the
+ * position table by an angle-sum step of 8 positions, so a rotated value can
+ * differ from dd_rope_qk's in its last bit (rarely). Outputs: o, lse and
+ * q_rot = R q, k_rot = R k (bf16, [B, L, H, d]), the q and k that dd_attn_bwd
+ * takes with rope_base > 0. Needs desc->rope_base > 0 and
+ * dd_attn_workspace_size(desc, 0) bytes of workspace (this call fills the
+ * table in it). q_rot may be q (in place); k_rot must not overlap k
+ * (DD_ERR_INVALID_ARG): work items still read k while others write k_rot. */
+dd_status dd_attn_fwd_rope(const dd_attn_desc* desc, const void* q, const void* k, const void* v, void* o,
+                           float* lse, void* q_rot, void* k_rot, void* ws, size_t ws_bytes, void* stream);
 
 /* Backward: from q, k, v, the forward's o and lse, and dO, writes dq, dk, dv
  * (bf16, overwritten, not accumulated). Recomputes P from lse. With

@@ -126,6 +126,76 @@ unsigned long long wait_limit_ns() {
   return v;
 }
 
+// Sequences of at most this many key tiles (L <= 512) have their K tiles rotated inside the
+// RoPE forward kernel: each K tile is loaded by at most two work items there. Longer ones
+// load each K tile in many items, so k is rotated once by a pass before the kernel (measured
+// per call at H = 16, d = 128, 65536 tokens: in-kernel K rotation 0.349 / 0.440 ms at
+// L = 256 / 512 against 0.376 / 0.466 with the pass; 1.353 against 1.061 at 4096).
+constexpr int kFwdRopeQKMaxTiles = 4;
+
+dd_status fwd_common(const dd_attn_desc* desc, const void* q, const void* k, const void* v, void* o, float* lse,
+                     void* q_rot, void* k_rot, void* ws, size_t ws_bytes, void* stream, bool fused_rope) {
+  dd_status st = check_desc(desc);
+  if (st != DD_OK) return st;
+  if (!q || !k || !v || !o || !lse) return DD_ERR_INVALID_ARG;
+  if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(o) || !aligned16(lse))
+    return DD_ERR_INVALID_ARG;
+  if (fused_rope) {
+    if (!has_rope(desc) || !q_rot || !k_rot || !aligned16(q_rot) || !aligned16(k_rot)) return DD_ERR_INVALID_ARG;
+    const uintptr_t kb = reinterpret_cast<uintptr_t>(k), kr = reinterpret_cast<uintptr_t>(k_rot);
+    const uintptr_t n = (uintptr_t)desc->B * desc->L * desc->H * desc->d * 2;
+    if (kr < kb + n && kb < kr + n) return DD_ERR_INVALID_ARG;  // k_rot must not overlap k
+  }
+  if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u) || ws_bytes < dd_attn_workspace_size(desc, 0))
+    return DD_ERR_WORKSPACE;
+  if ((st = check_device()) != DD_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const int nkt = (desc->L + 127) / 128;
+  const int rope = !fused_rope ? 0 : (nkt <= kFwdRopeQKMaxTiles ? 2 : 1);  // launch_attn_fwd's RoPE form
+  CUtensorMap tq, tk, tv;
+  if (!make_map(&tq, q, desc, 128) || !make_map(&tk, rope == 1 ? k_rot : k, desc, 128) ||
+      !make_map(&tv, v, desc, 128))
+    return DD_ERR_CUDA;
+  FwdParams p;
+  p.B = desc->B;
+  p.L = desc->L;
+  p.H = desc->H;
+  p.nqt = nkt;
+  p.scale_log2 = desc->scale * kLog2e;
+  p.offsets = desc->cu_doc_offsets;
+  p.n_offsets = desc->cu_doc_offsets ? desc->n_offsets : 0;
+  p.o = static_cast<__nv_bfloat16*>(o);
+  p.lse = lse;
+  p.status = static_cast<int*>(ws);
+  p.work_ctr = reinterpret_cast<unsigned int*>(static_cast<uint8_t*>(ws) + 64);  // inside the status block
+  p.timeout_ns = wait_limit_ns();
+  p.q_rot = static_cast<__nv_bfloat16*>(q_rot);
+  p.k_rot = static_cast<__nv_bfloat16*>(k_rot);
+  p.rope_rows = nullptr;
+  cudaError_t e = cudaSuccess;
+  if (fused_rope) {
+    float2* rows = reinterpret_cast<float2*>(static_cast<uint8_t*>(ws) + kStatusBytes);
+    p.rope_rows = rows;
+    const RopeFreq f = rope_freq(desc);
+    if ((e = launch_rope_table(desc->L, desc->d, f, nullptr, rows, s)) != cudaSuccess) return DD_ERR_CUDA;
+    if (rope == 1) {  // k -> k_rot in one pass; the kernel reads k_rot
+      RopeParams rp;
+      rp.rows = (long long)desc->B * desc->L;
+      rp.L = desc->L;
+      rp.H = desc->H;
+      rp.d = desc->d;
+      rp.q = nullptr;
+      rp.k = static_cast<const __nv_bfloat16*>(k);
+      rp.q_rot = nullptr;
+      rp.k_rot = static_cast<__nv_bfloat16*>(k_rot);
+      rp.f = f;
+      if ((e = launch_rope_qk(rp, s)) != cudaSuccess) return DD_ERR_CUDA;
+    }
+  }
+  e = launch_attn_fwd(desc->d, tq, tk, tv, p, rope, s);
+  return e == cudaSuccess ? DD_OK : DD_ERR_CUDA;
+}
+
 }  // namespace
 
 dd_status validate_desc(const dd_attn_desc* desc) { return check_desc(desc); }
@@ -153,7 +223,7 @@ extern "C" {
 
 size_t dd_attn_workspace_size(const dd_attn_desc* desc, int for_bwd) {
   if (check_desc(desc) != DD_OK) return 0;
-  if (!for_bwd) return kStatusBytes;
+  if (!for_bwd) return kStatusBytes + rope_rows_bytes(desc);  // + the RoPE forward's (cos, sin) rows
   return kStatusBytes + 2 * bwd_vec_bytes(desc) + bwd_acc_bytes(desc) + rope_tab_bytes(desc) + rope_rows_bytes(desc);
 }
 
@@ -180,32 +250,12 @@ dd_status dd_rope_qk(const dd_attn_desc* desc, const void* q, const void* k, voi
 
 dd_status dd_attn_fwd(const dd_attn_desc* desc, const void* q, const void* k, const void* v, void* o, float* lse,
                       void* ws, size_t ws_bytes, void* stream) {
-  dd_status st = check_desc(desc);
-  if (st != DD_OK) return st;
-  if (!q || !k || !v || !o || !lse) return DD_ERR_INVALID_ARG;
-  if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(o) || !aligned16(lse))
-    return DD_ERR_INVALID_ARG;
-  if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u) || ws_bytes < dd_attn_workspace_size(desc, 0))
-    return DD_ERR_WORKSPACE;
-  if ((st = check_device()) != DD_OK) return st;
-  CUtensorMap tq, tk, tv;
-  if (!make_map(&tq, q, desc, 128) || !make_map(&tk, k, desc, 128) || !make_map(&tv, v, desc, 128))
-    return DD_ERR_CUDA;
-  FwdParams p;
-  p.B = desc->B;
-  p.L = desc->L;
-  p.H = desc->H;
-  p.nqt = (desc->L + 127) / 128;
-  p.scale_log2 = desc->scale * kLog2e;
-  p.offsets = desc->cu_doc_offsets;
-  p.n_offsets = desc->cu_doc_offsets ? desc->n_offsets : 0;
-  p.o = static_cast<__nv_bfloat16*>(o);
-  p.lse = lse;
-  p.status = static_cast<int*>(ws);
-  p.work_ctr = reinterpret_cast<unsigned int*>(static_cast<uint8_t*>(ws) + 64);  // inside the status block
-  p.timeout_ns = wait_limit_ns();
-  cudaError_t e = launch_attn_fwd(desc->d, tq, tk, tv, p, static_cast<cudaStream_t>(stream));
-  return e == cudaSuccess ? DD_OK : DD_ERR_CUDA;
+  return fwd_common(desc, q, k, v, o, lse, nullptr, nullptr, ws, ws_bytes, stream, false);
+}
+
+dd_status dd_attn_fwd_rope(const dd_attn_desc* desc, const void* q, const void* k, const void* v, void* o,
+                           float* lse, void* q_rot, void* k_rot, void* ws, size_t ws_bytes, void* stream) {
+  return fwd_common(desc, q, k, v, o, lse, q_rot, k_rot, ws, ws_bytes, stream, true);
 }
 
 dd_status dd_attn_bwd(const dd_attn_desc* desc, const void* q, const void* k, const void* v, const void* o,

@@ -63,21 +63,35 @@ struct FwdCfg {
   static constexpr int OFF_K = OFF_Q + 2 * Q_BYTES;
   static constexpr int OFF_V = OFF_K + KST * KV_BYTES;
   static constexpr int OFF_BAR = OFF_V + VST * KV_BYTES;
-  static constexpr int SMEM_BYTES = OFF_BAR + 256 + 1024;
+  static constexpr int SMEM_BYTES = OFF_BAR + 512 + 1024;
   static constexpr int PF = 4;  // K / V tiles prefetched into L2 ahead of the ring
   static constexpr uint32_t TMEM_S = 0, TMEM_O = 256, TMEM_COLS = 512;
-  static constexpr int THREADS = 384;
-  // setmaxnreg split (the spill-free one for each head dim under ptxas 13.0)
+  static constexpr int THREADS = 384;  // the RoPE forms add a rotation warpgroup: 512
+  // setmaxnreg split (the spill-free one for each head dim under ptxas 13.0); REGS_ROT: the
+  // rotation warpgroup of the RoPE forms
   static constexpr int REGS_LOW = D == 128 ? 80 : 72, REGS_HIGH = D == 128 ? 184 : 192;
+  static constexpr int REGS_ROT = D == 128 ? 64 : 56;
 };
-// The split must fit in the launch's 384 threads x 168 registers.
+// The split must fit in the launch's 384 threads x 168 registers (512 x 128 with RoPE).
 static_assert(128 * FwdCfg<128>::REGS_LOW + 256 * FwdCfg<128>::REGS_HIGH <= 384 * 168, "register split");
 static_assert(128 * FwdCfg<64>::REGS_LOW + 256 * FwdCfg<64>::REGS_HIGH <= 384 * 168, "register split");
+static_assert(128 * (FwdCfg<128>::REGS_LOW + FwdCfg<128>::REGS_ROT) + 256 * FwdCfg<128>::REGS_HIGH <= 512 * 128,
+              "register split");
+static_assert(128 * (FwdCfg<64>::REGS_LOW + FwdCfg<64>::REGS_ROT) + 256 * FwdCfg<64>::REGS_HIGH <= 512 * 128,
+              "register split");
+
+// RoPE forms of the forward kernel: none (q, k given rotated, or no RoPE); Q tiles rotated in
+// shared memory as they land (k given rotated); Q and K tiles rotated as they land.
+enum FwdRope { kRopeNone = 0, kRopeQ = 1, kRopeQK = 2 };
+__host__ __device__ constexpr int fwd_threads(int rope) { return rope ? 512 : 384; }
+
 
 // The item ring: warp 11 claims each next item and publishes its index to the roles that
 // read it: the K and V producer lanes, the 32 lanes of the MMA warp and the 256 softmax
 // threads, each of which arrives on item_empty after reading.
-constexpr int kItemRing = 4, kItemReaders = 1 + 1 + 32 + 256;
+// The RoPE forms add the 128 rotation threads.
+constexpr int kItemRing = 4;
+__host__ __device__ constexpr int fwd_item_readers(int rope) { return 1 + 1 + 32 + 256 + (rope ? 128 : 0); }
 
 struct FwdBars {
   uint64_t item_full[kItemRing], item_empty[kItemRing];
@@ -86,10 +100,11 @@ struct FwdBars {
   uint64_t k_full[2], k_empty[2], v_full[2], v_empty[2];
   uint64_t s_full[2], p_full[2], pv_done[2];
   uint64_t mma_drain;
+  uint64_t q_rot[2], k_rot[2];  // RoPE forms: Q_t / the K stage has been rotated in shared memory
   uint32_t tmem_base;
   int abort_flag;
 };
-static_assert(sizeof(FwdBars) <= 256, "barrier block");
+static_assert(sizeof(FwdBars) <= 512, "barrier block");
 static_assert(FwdCfg<128>::KST == 2 && FwdCfg<128>::VST == 2, "ring barriers");
 
 // A work item: query tiles 2u and 2u + 1 of one (sequence, head). Items are numbered pair
@@ -152,8 +167,67 @@ __device__ __forceinline__ int fwd_next_item(FwdBars* bars, int n, bool& ok, con
   return it;
 }
 
+// RoPE of one 128-row tile in shared memory, in place: row r holds position pos0 + r and
+// each pair (x_2j, x_2j+1) becomes (x_2j c - x_2j+1 s, x_2j s + x_2j+1 c), c, s = cos, sin
+// of (pos0 + r) theta_j, in fp32, rounded to bf16 (rope_rotate_bf16x2, the arithmetic of
+// dd_rope_qk). Rows at or past L are TMA zero fill and stay as they are. With gdst set
+// the rotated rows below L are also written to global memory (gdst: element 0 of row pos0,
+// rows `rs` elements apart). Thread t of the 128 takes the 16-byte chunk c = t % 16
+// (columns 8c .. 8c + 7: pairs 4c .. 4c + 3) of rows g, g + 8, ..., g + 120 (g = t / 16),
+// which share one swizzled chunk position (the 128B swizzle XORs the chunk index with
+// row % 8 = g). Its (cos, sin) start from the table row of position pos0 + g (the values
+// dd_rope_qk uses) and advance eight positions per row by the angle-sum step with
+// (C, S) = (cos, sin) of 8 theta_j (table row 8): after up to 15 steps they are within a
+// few 1e-7 of the table's, so a rotated value can differ from dd_rope_qk's in its last bit
+// where the fp32 result lies that close to a bf16 rounding boundary (rare).
 template <int D>
-__global__ void __launch_bounds__(384, 1)
+__device__ __forceinline__ void rope_step8(const FwdParams& p, int t, float (&stc)[4], float (&sts)[4]) {
+  const int c = t & 15;
+#pragma unroll
+  for (int e = 0; e < 4; e++) {
+    stc[e] = 1.f;
+    sts[e] = 0.f;
+  }
+  if (p.L > 8 && c < D / 8) {  // with L <= 8 no thread steps past its first row
+#pragma unroll
+    for (int e = 0; e < 4; e++) {
+      const float2 v = __ldg(p.rope_rows + 8 * (D / 2) + 4 * c + e);
+      stc[e] = v.x;
+      sts[e] = v.y;
+    }
+  }
+}
+template <int D>
+__device__ __forceinline__ void rope_rotate_tile(uint8_t* tile, int pos0, int L, const float2* tab,
+                                                 const float (&stc)[4], const float (&sts)[4], __nv_bfloat16* gdst,
+                                                 long long rs, int t) {
+  const int c = t & 15, g = t >> 4;
+  if (c >= D / 8 || pos0 + g >= L) return;
+  const uint32_t base = smem_u32(tile) + (uint32_t)(c >> 3) * (128u * 128u) + sw128_offset((uint32_t)g, c & 7);
+  const float4* t4 = reinterpret_cast<const float4*>(tab + (long long)(pos0 + g) * (D / 2) + 4 * c);
+  const float4 a = __ldg(t4), b = __ldg(t4 + 1);
+  float cv[4] = {a.x, a.z, b.x, b.z}, sv[4] = {a.y, a.w, b.y, b.w};
+#pragma unroll 2
+  for (int k = 0; k < 16; k++) {
+    const int r = g + 8 * k;
+    if (pos0 + r >= L) break;
+    const uint32_t addr = base + (uint32_t)k * 1024u;  // eight rows on: the same swizzle phase
+    const float4 x4 = lds_f4(addr);
+    uint32_t w[4] = {__float_as_uint(x4.x), __float_as_uint(x4.y), __float_as_uint(x4.z), __float_as_uint(x4.w)};
+#pragma unroll
+    for (int e = 0; e < 4; e++) {
+      w[e] = rope_rotate_bf16x2(__uint_as_float(w[e] << 16), __uint_as_float(w[e] & 0xffff0000u), cv[e], sv[e]);
+      const float cn = fmaf(cv[e], stc[e], -sv[e] * sts[e]);
+      sv[e] = fmaf(sv[e], stc[e], cv[e] * sts[e]);
+      cv[e] = cn;
+    }
+    st_shared_v4(addr, w[0], w[1], w[2], w[3]);
+    if (gdst) *reinterpret_cast<uint4*>(gdst + r * rs + 8 * c) = make_uint4(w[0], w[1], w[2], w[3]);
+  }
+}
+
+template <int D, int ROPE>
+__global__ void __launch_bounds__(fwd_threads(ROPE), 1)
     attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                        const __grid_constant__ CUtensorMap tmV, const FwdParams p) {
   using C = FwdCfg<D>;
@@ -171,7 +245,7 @@ __global__ void __launch_bounds__(384, 1)
     bars->abort_flag = 0;
     for (int i = 0; i < kItemRing; i++) {
       mbar_init(&bars->item_full[i], 1);
-      mbar_init(&bars->item_empty[i], kItemReaders);
+      mbar_init(&bars->item_empty[i], fwd_item_readers(ROPE));
     }
     for (int t = 0; t < 2; t++) {
       mbar_init(&bars->q_full[t], 1);
@@ -185,6 +259,8 @@ __global__ void __launch_bounds__(384, 1)
       mbar_init(&bars->k_empty[i], 1);
       mbar_init(&bars->v_full[i], 1);
       mbar_init(&bars->v_empty[i], 1);
+      mbar_init(&bars->q_rot[i], 128);
+      mbar_init(&bars->k_rot[i], 128);
     }
     mbar_init(&bars->mma_drain, 1);
     fence_mbar_init();
@@ -319,8 +395,11 @@ __global__ void __launch_bounds__(384, 1)
           // S_t = Q_t K_j^T into the buffer PV_t has just read (issue order keeps them apart)
           if (ok && tile && j < NJ && kt >= lo_t && kt <= hi_t) {
             const int jk = jg0 + j;
-            ok = __all_sync(0xffffffffu, mbar_wait(&bars->k_full[jk & 1], (jk >> 1) & 1, wd) &&
-                                             (ns_i[t] > 0 || mbar_wait(&bars->q_full[t], nit[t] & 1, wd)));
+            // With RoPE the rotation warpgroup's q_rot / k_rot follow q_full / k_full.
+            uint64_t* kb = ROPE == kRopeQK ? &bars->k_rot[jk & 1] : &bars->k_full[jk & 1];
+            uint64_t* qb = ROPE ? &bars->q_rot[t] : &bars->q_full[t];
+            ok = __all_sync(0xffffffffu, mbar_wait(kb, (jk >> 1) & 1, wd) &&
+                                             (ns_i[t] > 0 || mbar_wait(qb, nit[t] & 1, wd)));
           }
           if (ok && tile && j < NJ && kt >= lo_t && kt <= hi_t) {
             const int ks = (jg0 + j) & 1;
@@ -349,6 +428,55 @@ __global__ void __launch_bounds__(384, 1)
       if (leader) umma_commit(&bars->mma_drain);
       __syncwarp();
       mbar_wait_drain(&bars->mma_drain, 0, wd.limit_ns);
+    }
+  }
+  } else if (ROPE && wg == 3) {
+  setmaxnreg_dec<C::REGS_ROT>();
+  // ---------------- rotation warpgroup (RoPE forms): in the order the MMA thread needs them,
+  // Q_0 of an item, its first key tile, Q_1, then its other key tiles (key tiles with
+  // kRopeQK only), each rotated in place as soon as its TMA copy has landed and released
+  // with q_rot / k_rot (fence.proxy.async first: the tensor core reads these generic-proxy
+  // writes). Every Q tile also goes to q_rot in global memory for the backward, and every
+  // key tile to k_rot from the one item on whose diagonal it lies (key tile 2u or 2u + 1 of
+  // item u).
+  {
+    const int t = threadIdx.x - 384;
+    float stc[4], sts[4];
+    rope_step8<D>(p, t, stc, sts);
+    const long long rs = (long long)p.H * D;  // elements between rows of q / k
+    int nq[2] = {0, 0}, jg = 0;
+    bool ok = true;
+    for (int n = 0; ok; n++) {
+      const int it = fwd_next_item(bars, n, ok, wd);
+      if (it < 0) break;
+      const FwdItem I = fwd_item(p, it);
+      const long long row_base = ((long long)I.b * p.L) * p.H + I.h;  // (b, position 0, h) in rows of d
+      // e = 0: Q_0; e = 1: key tile J0; e = 2: Q_1; e >= 3: key tile J0 + e - 2.
+      for (int e = 0; e < I.NJ + 2 && ok; e++) {
+        if (e == 0 || e == 2) {
+          const int tq = e / 2;
+          if (tq == 1 && !I.has1) continue;
+          if (!(ok = __all_sync(0xffffffffu, mbar_wait(&bars->q_full[tq], nq[tq] & 1, wd)))) break;
+          const int pos0 = (2 * I.u + tq) * C::BM;
+          rope_rotate_tile<D>(sQ + tq * C::Q_BYTES, pos0, p.L, p.rope_rows, stc, sts,
+                              p.q_rot + (row_base + (long long)pos0 * p.H) * D, rs, t);
+          fence_proxy_async_smem();
+          mbar_arrive(&bars->q_rot[tq]);
+          nq[tq]++;
+        } else if (ROPE == kRopeQK) {
+          const int jj = e == 1 ? 0 : e - 2;
+          const int jk = jg + jj;
+          if (!(ok = __all_sync(0xffffffffu, mbar_wait(&bars->k_full[jk & 1], (jk >> 1) & 1, wd)))) break;
+          const int kt = I.J0 + jj;
+          const int pos0 = kt * C::BN;
+          const bool diag = kt == 2 * I.u || (I.has1 && kt == 2 * I.u + 1);
+          rope_rotate_tile<D>(sK + (jk & 1) * C::KV_BYTES, pos0, p.L, p.rope_rows, stc, sts,
+                              diag ? p.k_rot + (row_base + (long long)pos0 * p.H) * D : nullptr, rs, t);
+          fence_proxy_async_smem();
+          mbar_arrive(&bars->k_rot[jk & 1]);
+        }
+      }
+      jg += I.NJ;
     }
   }
   } else {
@@ -509,13 +637,13 @@ __global__ void __launch_bounds__(384, 1)
   }
 }
 
-template <int D>
+template <int D, int ROPE>
 static cudaError_t launch_fwd_d(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
                                const FwdParams& p, cudaStream_t stream) {
   using C = FwdCfg<D>;
   static DeviceCache nsm_dev;
   int nsm = 0;
-  cudaError_t e = kernel_setup(nsm_dev, attn_fwd_kernel<D>, C::SMEM_BYTES, &nsm);
+  cudaError_t e = kernel_setup(nsm_dev, attn_fwd_kernel<D, ROPE>, C::SMEM_BYTES, &nsm);
   if (e != cudaSuccess) return e;
   // One CTA per SM (shared memory allows no more) walking items: the first G in order, the
   // rest claimed. G is kept coprime with the pairs per (sequence, head), so the first round
@@ -534,15 +662,23 @@ static cudaError_t launch_fwd_d(const CUtensorMap& tq, const CUtensorMap& tk, co
   };
   while (G > 1 && gcd(G, nqp) != 1) G--;
   if ((e = cudaMemsetAsync(p.work_ctr, 0, sizeof(unsigned int), stream)) != cudaSuccess) return e;  // the claim counter
-  attn_fwd_kernel<D><<<(unsigned)G, C::THREADS, C::SMEM_BYTES, stream>>>(tq, tk, tv, p);
+  attn_fwd_kernel<D, ROPE><<<(unsigned)G, fwd_threads(ROPE), C::SMEM_BYTES, stream>>>(tq, tk, tv, p);
   return cudaGetLastError();
 }
 
+template <int D>
+static cudaError_t launch_fwd_rope(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
+                                   const FwdParams& p, int rope, cudaStream_t stream) {
+  if (rope == kRopeQK) return launch_fwd_d<D, kRopeQK>(tq, tk, tv, p, stream);
+  if (rope == kRopeQ) return launch_fwd_d<D, kRopeQ>(tq, tk, tv, p, stream);
+  return launch_fwd_d<D, kRopeNone>(tq, tk, tv, p, stream);
+}
+
 cudaError_t launch_attn_fwd(int d, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
-                            const FwdParams& p, cudaStream_t stream) {
-  if (d == 64) return launch_fwd_d<64>(tq, tk, tv, p, stream);
-  if (d == 80) return launch_fwd_d<80>(tq, tk, tv, p, stream);
-  return launch_fwd_d<128>(tq, tk, tv, p, stream);
+                            const FwdParams& p, int rope, cudaStream_t stream) {
+  if (d == 64) return launch_fwd_rope<64>(tq, tk, tv, p, rope, stream);
+  if (d == 80) return launch_fwd_rope<80>(tq, tk, tv, p, rope, stream);
+  return launch_fwd_rope<128>(tq, tk, tv, p, rope, stream);
 }
 
 }  // namespace ddattn

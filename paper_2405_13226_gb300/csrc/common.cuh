@@ -93,6 +93,13 @@ __device__ __forceinline__ long long rope_tab_index(int m, int d, int jj) {
   return ((long long)(m >> 5) * (d / 4) + jj) * 32 + (m & 31);
 }
 
+// R x for one pair (x0, x1) = (x_2j, x_2j+1) with (c, s) = (cos, sin) of m theta_j, fp32,
+// rounded to a bf16 pair (first element in the low half). Every kernel that rotates q or k
+// uses this, so they agree bit for bit.
+__device__ __forceinline__ uint32_t rope_rotate_bf16x2(float x0, float x1, float c, float s) {
+  return pack_bf16x2(fmaf(x0, c, -x1 * s), fmaf(x0, s, x1 * c));
+}
+
 // g <- R^T g for one rotated pair (cs = (cos, sin)).
 __device__ __forceinline__ void rope_unrotate_pair(float& g0, float& g1, float c, float s) {
   const float a = fmaf(g0, c, g1 * s);
@@ -141,6 +148,12 @@ struct FwdParams {
   int* status;
   unsigned int* work_ctr;  // items claimed past the first G (in the workspace's status block, zeroed per launch)
   unsigned long long timeout_ns;
+  // RoPE forms only: rotated q / k written for the backward (with K tiles not rotated in
+  // the kernel, k_rot is the k it reads, rotated by a pass before it), and the (cos, sin)
+  // of m theta_j row-major [L, d/2] (in the workspace, filled before the kernel).
+  __nv_bfloat16* q_rot;
+  __nv_bfloat16* k_rot;
+  const float2* rope_rows;
 };
 
 struct BwdParams {
@@ -168,7 +181,7 @@ struct BwdParams {
 struct RopeParams {
   long long rows;  // B * L token rows
   int L, H, d;
-  const __nv_bfloat16* q;
+  const __nv_bfloat16* q;  // nullptr: rotate k only
   const __nv_bfloat16* k;
   __nv_bfloat16* q_rot;
   __nv_bfloat16* k_rot;
@@ -207,8 +220,9 @@ inline cudaError_t kernel_setup(DeviceCache& nsm, Kernel kernel, int smem_bytes,
 dd_status validate_desc(const dd_attn_desc* desc);
 
 // Launchers (defined in attn_fwd.cu / attn_bwd.cu / rope.cu); return a cudaError_t.
+// rope: 0 none; 1 the kernel rotates its Q tiles (k given rotated); 2 it rotates Q and K tiles.
 cudaError_t launch_attn_fwd(int d, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
-                            const FwdParams& p, cudaStream_t stream);
+                            const FwdParams& p, int rope, cudaStream_t stream);
 cudaError_t launch_attn_bwd_main_d128(int d, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
                                       const CUtensorMap& tdo, const BwdParams& p, cudaStream_t stream);
 cudaError_t launch_attn_bwd_main_d128_persist(int d, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,

@@ -32,7 +32,7 @@ __global__ void __launch_bounds__(kThreads) rope_qk_kernel(const __grid_constant
   __syncthreads();
   const int vpr = p.H * p.d / 8;        // 16-byte vectors per token row
   const int per_tensor = nrows * vpr;
-  const int total = 2 * per_tensor;
+  const int total = (p.q ? 2 : 1) * per_tensor;  // q == nullptr: k only
   const long long base = r0 * p.H * p.d;
   for (int t0 = threadIdx.x; t0 < total; t0 += kThreads * kBatch) {
     uint4 x[kBatch];
@@ -40,8 +40,8 @@ __global__ void __launch_bounds__(kThreads) rope_qk_kernel(const __grid_constant
     for (int u = 0; u < kBatch; u++) {
       const int t = t0 + u * kThreads;
       if (t < total) {
-        const bool is_k = t >= per_tensor;
-        const int idx = is_k ? t - per_tensor : t;
+        const bool is_k = !p.q || t >= per_tensor;
+        const int idx = (p.q && is_k) ? t - per_tensor : t;
         const uint4* src = reinterpret_cast<const uint4*>((is_k ? p.k : p.q) + base) + idx;
         x[u] = __ldcs(src);   // read once: streaming
       }
@@ -50,8 +50,8 @@ __global__ void __launch_bounds__(kThreads) rope_qk_kernel(const __grid_constant
     for (int u = 0; u < kBatch; u++) {
       const int t = t0 + u * kThreads;
       if (t < total) {
-        const bool is_k = t >= per_tensor;
-        const int idx = is_k ? t - per_tensor : t;
+        const bool is_k = !p.q || t >= per_tensor;
+        const int idx = (p.q && is_k) ? t - per_tensor : t;
         const int rr = idx / vpr;
         const int col = ((idx - rr * vpr) * 8) % p.d;   // head-local column of the first element
         const float2* c = &cs[rr][col >> 1];
@@ -60,7 +60,7 @@ __global__ void __launch_bounds__(kThreads) rope_qk_kernel(const __grid_constant
         for (int e = 0; e < 4; e++) {
           const float2 v = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w[e]));
           const float2 r = c[e];
-          w[e] = pack_bf16x2(fmaf(v.x, r.x, -v.y * r.y), fmaf(v.x, r.y, v.y * r.x));
+          w[e] = rope_rotate_bf16x2(v.x, v.y, r.x, r.y);
         }
         uint4* dst = reinterpret_cast<uint4*>((is_k ? p.k_rot : p.q_rot) + base) + idx;
         __stcs(dst, make_uint4(w[0], w[1], w[2], w[3]));
@@ -70,7 +70,7 @@ __global__ void __launch_bounds__(kThreads) rope_qk_kernel(const __grid_constant
 }
 
 // One thread per (position m, pair-pair jj): two (cos, sin) values into the
-// float4 of rope_tab_index(m, d, jj) and into the row-major copy.
+// float4 of rope_tab_index(m, d, jj) (unless tab is null) and into the row-major copy.
 __global__ void __launch_bounds__(256) rope_table_kernel(int L, int d, const __grid_constant__ RopeFreq f,
                                                          float4* tab, float2* tab_rows) {
   const int quarter = d / 4;
@@ -79,7 +79,7 @@ __global__ void __launch_bounds__(256) rope_table_kernel(int L, int d, const __g
     const int m = (int)(t / quarter), jj = (int)(t % quarter);
     const float2 a = rope_cos_sin(m, f.hi[2 * jj], f.lo[2 * jj]);
     const float2 b = rope_cos_sin(m, f.hi[2 * jj + 1], f.lo[2 * jj + 1]);
-    tab[rope_tab_index(m, d, jj)] = make_float4(a.x, a.y, b.x, b.y);
+    if (tab) tab[rope_tab_index(m, d, jj)] = make_float4(a.x, a.y, b.x, b.y);
     reinterpret_cast<float4*>(tab_rows)[t] = make_float4(a.x, a.y, b.x, b.y);  // = [m][2jj], [m][2jj+1]
   }
 }

@@ -34,8 +34,8 @@ class Desc(ctypes.Structure):
 
 _lib = None
 
-EXPORTS = ("dd_attn_workspace_size", "dd_attn_fwd", "dd_attn_bwd", "dd_attn_bwd_phases", "dd_attn_bwd_noalloc",
-           "dd_rope_qk", "dd_attn_clear_status", "dd_attn_poll_status", "dd_selftest_wait_timeout",
+EXPORTS = ("dd_attn_workspace_size", "dd_attn_fwd", "dd_attn_fwd_rope", "dd_attn_bwd", "dd_attn_bwd_phases",
+           "dd_attn_bwd_noalloc", "dd_rope_qk", "dd_attn_clear_status", "dd_attn_poll_status", "dd_selftest_wait_timeout",
            "dd_status_string")
 NOALLOC_SCRATCH_BYTES = 32 << 20
 DD_BWD_PRE, DD_BWD_MAIN, DD_BWD_POST, DD_BWD_ALL = 1, 2, 4, 7
@@ -55,6 +55,8 @@ def lib() -> ctypes.CDLL:
         L.dd_attn_workspace_size.restype = sz
         L.dd_attn_fwd.argtypes = [dp, vp, vp, vp, vp, vp, vp, sz, vp]
         L.dd_attn_fwd.restype = i32
+        L.dd_attn_fwd_rope.argtypes = [dp, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]
+        L.dd_attn_fwd_rope.restype = i32
         L.dd_attn_bwd.argtypes = [dp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]
         L.dd_attn_bwd.restype = i32
         L.dd_attn_bwd_phases.argtypes = [dp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, i32, vp]
@@ -148,6 +150,29 @@ def fwd(q, k, v, scale=None, cu_doc_offsets=None, out=None, lse=None, workspace=
     if st != DD_OK:
         raise DDAttnError(st, "dd_attn_fwd")
     return out, lse
+
+
+def fwd_rope(q, k, v, rope_base, scale=None, cu_doc_offsets=None, out=None, lse=None, q_rot=None, k_rot=None,
+             workspace=None, stream=None):
+    """o, lse, q_rot, k_rot = attention forward with RoPE (base rope_base) applied
+    inside the kernel to the un-rotated q, k; q_rot, k_rot are the rotated
+    tensors the backward takes (bwd(..., rope_base=rope_base))."""
+    _check_qkv(q, k, v)
+    B, L, H, d = q.shape
+    desc = make_desc(B, L, H, d, scale, cu_doc_offsets, rope_base)
+    out = torch.empty_like(q) if out is None else out
+    lse = torch.empty((B, H, L), dtype=torch.float32, device=q.device) if lse is None else lse
+    q_rot = torch.empty_like(q) if q_rot is None else q_rot
+    k_rot = torch.empty_like(k) if k_rot is None else k_rot
+    _check_qkv(q_rot, k_rot)
+    if workspace is None:
+        workspace = new_workspace(desc, q.device, for_bwd=False)
+    st = lib().dd_attn_fwd_rope(ctypes.byref(desc), q.data_ptr(), k.data_ptr(), v.data_ptr(), out.data_ptr(),
+                                lse.data_ptr(), q_rot.data_ptr(), k_rot.data_ptr(), workspace.data_ptr(),
+                                workspace.numel(), _stream(stream))
+    if st != DD_OK:
+        raise DDAttnError(st, "dd_attn_fwd_rope")
+    return out, lse, q_rot, k_rot
 
 
 def bwd(q, k, v, o, dO, lse, scale=None, cu_doc_offsets=None, dq=None, dk=None, dv=None, workspace=None,

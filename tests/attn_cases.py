@@ -39,9 +39,11 @@ def bits_f64(bits) -> np.ndarray:
     return wl.bf16_bits_to_f32(bits).astype(np.float64)
 
 
-def run_cuda(qb, kb, vb, gb, scale, offsets=None, device="cuda", rope_base=0.0):
+def run_cuda(qb, kb, vb, gb, scale, offsets=None, device="cuda", rope_base=0.0, fused_rope=False, rotated=None):
     """fwd + bwd through the C ABI on bf16 bit arrays [B, L, H, d] (with
-    rope_base > 0: rope_qk first, and dq, dk with respect to the un-rotated q, k)."""
+    rope_base > 0: rope_qk first, or with fused_rope the forward that rotates q, k
+    itself; dq, dk with respect to the un-rotated q, k). `rotated`, a list, receives
+    the fused forward's q_rot, k_rot."""
     import torch
     from paper_2405_13226_gb300 import ddattn
     q, k, v, g = (to_device(x, device) for x in (qb, kb, vb, gb))
@@ -49,9 +51,14 @@ def run_cuda(qb, kb, vb, gb, scale, offsets=None, device="cuda", rope_base=0.0):
     B, L, H, d = q.shape
     desc = ddattn.make_desc(B, L, H, d, scale, off, rope_base)
     ws = ddattn.new_workspace(desc, q.device, for_bwd=True)
-    if rope_base:
+    if rope_base and fused_rope:
+        o, lse, q, k = ddattn.fwd_rope(q, k, v, rope_base, scale, off, workspace=ws)
+        if rotated is not None:
+            rotated += [q, k]
+    elif rope_base:
         q, k = ddattn.rope_qk(q, k, rope_base)
-    o, lse = ddattn.fwd(q, k, v, scale, off, workspace=ws)
+    if not (rope_base and fused_rope):
+        o, lse = ddattn.fwd(q, k, v, scale, off, workspace=ws)
     dq, dk, dv = ddattn.bwd(q, k, v, o, g, lse, scale, off, workspace=ws, rope_base=rope_base)
     torch.cuda.synchronize()
     st = ddattn.poll_status(ws)
@@ -81,8 +88,9 @@ def oracle_full(qb, kb, vb, gb, scale, offsets=None, rope_base=0.0):
     return back(o), lse.reshape(B, H, L), dq, dk, back(dv)
 
 
-def check_full(qb, kb, vb, gb, scale, offsets=None, rope_base=0.0):
-    o, lse, dq, dk, dv = run_cuda(qb, kb, vb, gb, scale, offsets, rope_base=rope_base)
+def check_full(qb, kb, vb, gb, scale, offsets=None, rope_base=0.0, fused_rope=False, rotated=None):
+    o, lse, dq, dk, dv = run_cuda(qb, kb, vb, gb, scale, offsets, rope_base=rope_base, fused_rope=fused_rope,
+                                  rotated=rotated)
     ro, rlse, rdq, rdk, rdv = oracle_full(qb, kb, vb, gb, scale, offsets, rope_base)
     go = to_f64(o)
     errs = {
@@ -107,10 +115,11 @@ def sample_rows(L: int, n_rand: int, seed: int) -> np.ndarray:
     return np.array(sorted({r for r in fixed + rnd if 0 <= r < L}), dtype=np.int32)
 
 
-def check_sampled(qb, kb, vb, gb, scale, slices, offsets=None, n_rand=8, gpu=None, rope_base=0.0):
+def check_sampled(qb, kb, vb, gb, scale, slices, offsets=None, n_rand=8, gpu=None, rope_base=0.0,
+                  fused_rope=False):
     """Full-size GPU run (or `gpu` results), oracle on sampled rows of (b, h) slices."""
     if gpu is None:
-        gpu = run_cuda(qb, kb, vb, gb, scale, offsets, rope_base=rope_base)
+        gpu = run_cuda(qb, kb, vb, gb, scale, offsets, rope_base=rope_base, fused_rope=fused_rope)
     o, lse, dq, dk, dv = (to_f64(t) for t in gpu)
     B, L, H, d = qb.shape
     acc = {k: ([], []) for k in ("o", "lse", "dq", "dk", "dv")}

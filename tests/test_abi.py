@@ -88,7 +88,9 @@ def test_rope_descriptor_and_workspace(lib):
     tab = (224 * 64 * 8 + 255) // 256 * 256        # warp-blocked layout, positions rounded up to 32
     tab += (200 * 64 * 8 + 255) // 256 * 256       # row-major copy
     assert lib.workspace_size(roped, True) == lib.workspace_size(plain, True) + tab
-    assert lib.workspace_size(roped, False) == 256
+    # the fused-RoPE forward keeps the row-major table in its workspace
+    assert lib.workspace_size(roped, False) == 256 + (200 * 64 * 8 + 255) // 256 * 256
+    assert lib.workspace_size(plain, False) == 256
     for bad in (-1.0, float("nan"), float("inf")):
         assert lib.workspace_size(lib.make_desc(3, 200, 2, 128, rope_base=bad), True) == 0
 
@@ -127,3 +129,27 @@ def test_noalloc_bad_descriptor_codes_match_bwd(lib):
     unsupported = lib.make_desc(2, 256, 2, 96)
     assert L.dd_attn_bwd_noalloc(ctypes.byref(unsupported), *p, None, None) == lib.DD_ERR_UNSUPPORTED
     assert L.dd_attn_bwd_noalloc(None, *p, None, None) == lib.DD_ERR_INVALID_ARG
+
+
+def test_fwd_rope_host_validation(lib):
+    """dd_attn_fwd_rope needs rope_base > 0, both rotated outputs, 16-byte alignment and a
+    k_rot that does not overlap k (work items still read k while others write k_rot);
+    q_rot may be q."""
+    L = lib.lib()
+    B, S, H, d = 2, 256, 2, 128
+    n = B * S * H * d * 2
+    q, k, v, o, lse, qr, kr = 0x1000000, 0x2000000, 0x3000000, 0x4000000, 0x5000000, 0x6000000, 0x7000000
+    desc = lib.make_desc(B, S, H, d, rope_base=1e4)
+    call = lambda dsc, ptrs, ws=None, wsb=0: L.dd_attn_fwd_rope(ctypes.byref(dsc), *ptrs, ws, wsb, None)
+    good = [q, k, v, o, lse, qr, kr]
+    assert call(lib.make_desc(B, S, H, d), good) == lib.DD_ERR_INVALID_ARG           # rope_base = 0
+    assert call(desc, good[:5] + [None, kr]) == lib.DD_ERR_INVALID_ARG               # no q_rot
+    assert call(desc, good[:6] + [None]) == lib.DD_ERR_INVALID_ARG                   # no k_rot
+    assert call(desc, good[:6] + [kr + 8]) == lib.DD_ERR_INVALID_ARG                 # misaligned k_rot
+    assert call(desc, good[:6] + [k]) == lib.DD_ERR_INVALID_ARG                      # k_rot is k
+    assert call(desc, good[:6] + [k + n - 16]) == lib.DD_ERR_INVALID_ARG             # overlaps k's end
+    assert call(desc, good[:6] + [k - n + 16]) == lib.DD_ERR_INVALID_ARG             # overlaps k's start
+    # k_rot right after k, q_rot in place: the arguments pass, then the workspace is checked
+    assert call(desc, good[:5] + [q, k + n]) == lib.DD_ERR_WORKSPACE
+    assert call(desc, good, 0x100000, 256) == lib.DD_ERR_WORKSPACE                  # no room for the table
+    assert call(lib.make_desc(B, S, H, 96, rope_base=1e4), good) == lib.DD_ERR_UNSUPPORTED
