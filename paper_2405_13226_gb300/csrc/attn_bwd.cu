@@ -242,13 +242,13 @@ __global__ void __launch_bounds__(320, 1)
       mbar_init(&bars->q_empty[i], 1);
     }
     mbar_init(&bars->s_full, 1);
-    mbar_init(&bars->sdp_free, 128);
-    mbar_init(&bars->p_full, 128);
+    mbar_init(&bars->sdp_free, 4);  // per-warp arrivals (mbar_arrive_warp)
+    mbar_init(&bars->p_full, 4);
     mbar_init(&bars->p_free, 1);
-    mbar_init(&bars->ds_full, 128);
+    mbar_init(&bars->ds_full, 4);
     mbar_init(&bars->ds_free, 1);
     mbar_init(&bars->dq_full, 1);
-    mbar_init(&bars->dq_free, 128);
+    mbar_init(&bars->dq_free, 4);
     mbar_init(&bars->mma_done, 1);
     fence_mbar_init();
   }
@@ -437,9 +437,9 @@ __global__ void __launch_bounds__(320, 1)
       // S^T / dP^T fully read; P^T and dS^T written.
       fence_proxy_async_smem();
       tc_fence_before();
-      mbar_arrive(&bars->sdp_free);
-      mbar_arrive(&bars->p_full);
-      mbar_arrive(&bars->ds_full);
+      mbar_arrive_warp(&bars->sdp_free);
+      mbar_arrive_warp(&bars->p_full);
+      mbar_arrive_warp(&bars->ds_full);
     }
     // Epilogue: dV rows.
     if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&bars->mma_done, 0, wd));
@@ -479,7 +479,7 @@ __global__ void __launch_bounds__(320, 1)
         tmem_ld_wait(v0);
         tmem_ld_wait(v1);
         tc_fence_before();
-        mbar_arrive(&bars->dq_free);
+        mbar_arrive_warp(&bars->dq_free);
       }
       if (t == 0) bulk_wait_read<0>();  // previous reduction has read the staging tile
       named_bar_sync(1, 128);

@@ -87,12 +87,12 @@ __global__ void __launch_bounds__(512, 1)
     }
     mbar_init(&bars->s_full, 1);
     mbar_init(&bars->dp_full, 1);
-    mbar_init(&bars->p_full, 256);
-    mbar_init(&bars->dp_read, 256);
-    mbar_init(&bars->dss_full, 256);
+    mbar_init(&bars->p_full, 8);  // per-warp arrivals (mbar_arrive_warp)
+    mbar_init(&bars->dp_read, 8);
+    mbar_init(&bars->dss_full, 8);
     mbar_init(&bars->dv_done, 1);
     mbar_init(&bars->dq_full, 1);
-    mbar_init(&bars->r_free, 128);
+    mbar_init(&bars->r_free, 4);
     mbar_init(&bars->mma_done, 1);
     fence_mbar_init();
   }
@@ -326,7 +326,7 @@ __global__ void __launch_bounds__(512, 1)
       tmem_st32(tl + rA + wg * 64, pk);
       tmem_st_wait();
       tc_fence_before();
-      mbar_arrive(&bars->p_full);
+      mbar_arrive_warp(&bars->p_full);
       // dS^T = P^T (dP^T - D), from the bf16 P^T that dV also uses.
       ok = __all_sync(0xffffffffu, mbar_wait(&bars->dp_full, i & 1, wd));
       if (!ok) break;
@@ -339,7 +339,7 @@ __global__ void __launch_bounds__(512, 1)
         tmem_ld_wait(d0);
         tmem_ld_wait(d1);
         tc_fence_before();
-        mbar_arrive(&bars->dp_read);  // region B may take S^T of the next step
+        mbar_arrive_warp(&bars->dp_read);  // region B may take S^T of the next step
 #pragma unroll
         for (int c = 0; c < 2; c++) {
           const uint32_t* dv = c ? d1 : d0;
@@ -371,7 +371,7 @@ __global__ void __launch_bounds__(512, 1)
       fence_proxy_async_smem();
       tmem_st_wait();
       tc_fence_before();
-      mbar_arrive(&bars->dss_full);
+      mbar_arrive_warp(&bars->dss_full);
     }
     // Epilogue: dV rows.
     if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&bars->mma_done, 0, wd));
@@ -413,7 +413,7 @@ __global__ void __launch_bounds__(512, 1)
 #pragma unroll
       for (int c = 0; c < 4; c++) tmem_ld_wait(v[c]);
       tc_fence_before();
-      mbar_arrive(&bars->r_free);
+      mbar_arrive_warp(&bars->r_free);
       const int q0 = (m_lo + i) * BQ;
       if (!drains) continue;
 #pragma unroll

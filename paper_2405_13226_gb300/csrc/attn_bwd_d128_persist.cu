@@ -81,16 +81,16 @@ __global__ void __launch_bounds__(512, 1)
     }
     mbar_init(&bars->s_full, 1);
     mbar_init(&bars->dp_full, 1);
-    mbar_init(&bars->p_full, 256);
-    mbar_init(&bars->dp_read, 256);
-    mbar_init(&bars->dss_full, 256);
+    mbar_init(&bars->p_full, 8);  // per-warp arrivals (mbar_arrive_warp)
+    mbar_init(&bars->dp_read, 8);
+    mbar_init(&bars->dss_full, 8);
     mbar_init(&bars->dv_done, 1);
     mbar_init(&bars->dq_full, 1);
-    mbar_init(&bars->r_free, 128);
+    mbar_init(&bars->r_free, 4);
     mbar_init(&bars->mma_done, 1);
     mbar_init(&bars->kv_empty, 1);
-    mbar_init(&bars->dv_free, 256);
-    mbar_init(&bars->dk_free, 128);
+    mbar_init(&bars->dv_free, 8);
+    mbar_init(&bars->dk_free, 4);
     mbar_init(&bars->mma_drain, 1);
     fence_mbar_init();
   }
@@ -360,7 +360,7 @@ __global__ void __launch_bounds__(512, 1)
       tmem_st32(tl + rA + wg * 64, pk);
       tmem_st_wait();
       tc_fence_before();
-      mbar_arrive(&bars->p_full);
+      mbar_arrive_warp(&bars->p_full);
       // dS^T = P^T (dP^T - D), from the bf16 P^T that dV also uses.
       ok = __all_sync(0xffffffffu, mbar_wait(&bars->dp_full, g & 1, wd));
       if (!ok) break;
@@ -373,7 +373,7 @@ __global__ void __launch_bounds__(512, 1)
         tmem_ld_wait(d0);
         tmem_ld_wait(d1);
         tc_fence_before();
-        mbar_arrive(&bars->dp_read);  // region B may take S^T of the next step
+        mbar_arrive_warp(&bars->dp_read);  // region B may take S^T of the next step
 #pragma unroll
         for (int c = 0; c < 2; c++) {
           const uint32_t* dv = c ? d1 : d0;
@@ -405,7 +405,7 @@ __global__ void __launch_bounds__(512, 1)
       fence_proxy_async_smem();
       tmem_st_wait();
       tc_fence_before();
-      mbar_arrive(&bars->dss_full);
+      mbar_arrive_warp(&bars->dss_full);
     }
     // Epilogue: dV rows of this item.
     if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&bars->mma_done, ic & 1, wd));
@@ -427,7 +427,7 @@ __global__ void __launch_bounds__(512, 1)
         }
       }
       tc_fence_before();
-      mbar_arrive(&bars->dv_free);  // dV of this item has left TMEM
+      mbar_arrive_warp(&bars->dv_free);  // dV of this item has left TMEM
     }
     g0 += nq;
     }
@@ -461,7 +461,7 @@ __global__ void __launch_bounds__(512, 1)
 #pragma unroll
       for (int c = 0; c < 4; c++) tmem_ld_wait(v[c]);
       tc_fence_before();
-      mbar_arrive(&bars->r_free);
+      mbar_arrive_warp(&bars->r_free);
       const int q0 = (m_lo + i) * BQ;
       if (!drains) continue;
 #pragma unroll
@@ -506,7 +506,7 @@ __global__ void __launch_bounds__(512, 1)
           store_dk_row32(dst + c * 32, v, p.scale, p.rope_tab, kv, D, c * 8, D - c * 32 < 32 ? D - c * 32 : 32);
       }
       tc_fence_before();
-      mbar_arrive(&bars->dk_free);  // dK of this item has left TMEM
+      mbar_arrive_warp(&bars->dk_free);  // dK of this item has left TMEM
     }
     // dQ owned: the query tiles whose last contributor is this key tile are complete once
     // this warp's copies have landed; convert its chunk of their rows to bf16 dq.

@@ -251,7 +251,7 @@ __global__ void __launch_bounds__(fwd_threads(ROPE), 1)
       mbar_init(&bars->q_full[t], 1);
       mbar_init(&bars->q_empty[t], 1);
       mbar_init(&bars->s_full[t], 1);
-      mbar_init(&bars->p_full[t], 128);
+      mbar_init(&bars->p_full[t], 4);  // per-warp arrivals (mbar_arrive_warp)
       mbar_init(&bars->pv_done[t], 1);
     }
     for (int i = 0; i < 2; i++) {
@@ -259,8 +259,8 @@ __global__ void __launch_bounds__(fwd_threads(ROPE), 1)
       mbar_init(&bars->k_empty[i], 1);
       mbar_init(&bars->v_full[i], 1);
       mbar_init(&bars->v_empty[i], 1);
-      mbar_init(&bars->q_rot[i], 128);
-      mbar_init(&bars->k_rot[i], 128);
+      mbar_init(&bars->q_rot[i], 4);
+      mbar_init(&bars->k_rot[i], 4);
     }
     mbar_init(&bars->mma_drain, 1);
     fence_mbar_init();
@@ -461,7 +461,7 @@ __global__ void __launch_bounds__(fwd_threads(ROPE), 1)
           rope_rotate_tile<D>(sQ + tq * C::Q_BYTES, pos0, p.L, p.rope_rows, stc, sts,
                               p.q_rot + (row_base + (long long)pos0 * p.H) * D, rs, t);
           fence_proxy_async_smem();
-          mbar_arrive(&bars->q_rot[tq]);
+          mbar_arrive_warp(&bars->q_rot[tq]);
           nq[tq]++;
         } else if (ROPE == kRopeQK) {
           const int jj = e == 1 ? 0 : e - 2;
@@ -473,7 +473,7 @@ __global__ void __launch_bounds__(fwd_threads(ROPE), 1)
           rope_rotate_tile<D>(sK + (jk & 1) * C::KV_BYTES, pos0, p.L, p.rope_rows, stc, sts,
                               diag ? p.k_rot + (row_base + (long long)pos0 * p.H) * D : nullptr, rs, t);
           fence_proxy_async_smem();
-          mbar_arrive(&bars->k_rot[jk & 1]);
+          mbar_arrive_warp(&bars->k_rot[jk & 1]);
         }
       }
       jg += I.NJ;
@@ -545,9 +545,17 @@ __global__ void __launch_bounds__(fwd_threads(ROPE), 1)
         if (kv > row || kv < ds) sc[c] = -INFINITY;
       }
     }
-    float mx = sc[0];
+    // Row max as eight independent 3-input max chains over 16 columns each, then a tree:
+    // the critical path is ~10 dependent instructions instead of a 127-long chain.
+    float mq[8];
 #pragma unroll
-    for (int c = 1; c < 128; c++) mx = fmaxf(mx, sc[c]);
+    for (int q = 0; q < 8; q++) {
+      float m = fmax3(sc[16 * q], sc[16 * q + 1], sc[16 * q + 2]);
+#pragma unroll
+      for (int e = 3; e < 15; e += 2) m = fmax3(m, sc[16 * q + e], sc[16 * q + e + 1]);
+      mq[q] = fmaxf(m, sc[16 * q + 15]);
+    }
+    const float mx = fmax3(fmax3(mq[0], mq[1], mq[2]), fmax3(mq[3], mq[4], mq[5]), fmaxf(mq[6], mq[7]));
     const float m_tile = mx * sl2;
     float alpha = 1.f;
     bool rescale = false;
@@ -558,18 +566,19 @@ __global__ void __launch_bounds__(fwd_threads(ROPE), 1)
     }
     const float m_use = (m_run == -INFINITY) ? 0.f : m_run;
     const uint64_t negm = f32x2(-m_use, -m_use);
-    uint64_t rs2 = f32x2(0.f, 0.f);
+    uint64_t rs2[4] = {f32x2(0.f, 0.f), f32x2(0.f, 0.f), f32x2(0.f, 0.f), f32x2(0.f, 0.f)};  // 4 sum chains
     uint32_t pk0[32], pk1[32];
 #pragma unroll
     for (int c = 0; c < 64; c++) {
       const uint64_t x = fma_f32x2(f32x2(sc[2 * c], sc[2 * c + 1]), sl2x2, negm);
       const float p0 = exp2_approx(f32x2_lo(x));
       const float p1 = exp2_approx(f32x2_hi(x));
-      rs2 = add_f32x2(rs2, f32x2(p0, p1));
+      rs2[c & 3] = add_f32x2(rs2[c & 3], f32x2(p0, p1));
       if (c < 32) pk0[c] = pack_bf16x2(p0, p1);
       else pk1[c - 32] = pack_bf16x2(p0, p1);
     }
-    l_run = l_run * alpha + (f32x2_lo(rs2) + f32x2_hi(rs2));
+    const uint64_t rsum = add_f32x2(add_f32x2(rs2[0], rs2[1]), add_f32x2(rs2[2], rs2[3]));
+    l_run = l_run * alpha + (f32x2_lo(rsum) + f32x2_hi(rsum));
     tmem_st32(sbuf + 0, pk0);
     tmem_st32(sbuf + 32, pk1);
     // O_t *= alpha. PV_t of the previous key tile has completed: it was issued
@@ -587,7 +596,7 @@ __global__ void __launch_bounds__(fwd_threads(ROPE), 1)
     }
     tmem_st_wait();
     tc_fence_before();
-    mbar_arrive(&bars->p_full[t]);
+    mbar_arrive_warp(&bars->p_full[t]);
   }
   // Epilogue: O / l -> bf16, LSE = (m + log2 l) * ln2.
   if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&bars->pv_done[t], nit & 1, wd));
