@@ -50,7 +50,7 @@ def kernel_source_sha1() -> str:
 def measured_traffic():
     """Mean DRAM bytes per launch of the backward main kernel over the sweep,
     from the committed ncu summary, if it was taken on the current sources."""
-    p = os.path.join(ROOT, "profiles", "attn_main_kernels_sweep_traffic.md")
+    p = os.path.join(ROOT, "profiles", "attn_kernels_sweep_traffic.md")
     if not os.path.exists(p):
         return None
     txt = open(p).read()
@@ -346,10 +346,10 @@ def run_ours(args):
     peak = peaks["bf16_tflops_sustained"]
     roofline = {"kernel": "attn_bwd_main (d=128: walking kernel for L <= 2048, per-key-tile kernel above)", "bound": "tensor", "achieved": main_ach, "peak": peak,
                 "unit": "TFLOP/s", "frac": main_ach / peak, "traffic": measured_traffic(),
-                "traffic_note": "not measured in this run: mean dram__bytes_read+write per launch over the six "
-                                "buckets, read from the committed ncu summary "
-                                "profiles/attn_main_kernels_sweep_traffic.md (one kernel and one launch per "
-                                "capture), keyed by a hash of the kernel sources; null if they changed since",
+                "traffic_note": "read from profiles/attn_kernels_sweep_traffic.md, not measured in this run: "
+                                "mean dram__bytes_read+write per launch over the six buckets from an ncu "
+                                "capture of this kernel alone (its first six launches), taken on the sources "
+                                "whose hash that file records; null if the sources changed since",
                 "peak_kind": "bf16_tflops_sustained (%s)" % peak_src,
                 "share_of_step": main_t / total_ms,
                 "fwd_kernel_tflops": sum(bk.flops_fwd for bk in buckets) * args.steps / (fwd_t * 1e-3) / 1e12,
