@@ -20,7 +20,7 @@ def lib():
 def _declared():
     src = open(os.path.join(ROOT, "include", "ddattn.h")).read()
     src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
-    return sorted(set(re.findall(r"\b(dd_[a-z_]+)\s*\(", src)))
+    return sorted(set(re.findall(r"\b(dd_[a-z0-9_]+)\s*\(", src)))
 
 
 def test_exports_every_declared_symbol(lib):
