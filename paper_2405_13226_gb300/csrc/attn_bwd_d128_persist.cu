@@ -411,29 +411,17 @@ __global__ void __launch_bounds__(512, 1)
     if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&bars->mma_done, ic & 1, wd));
     if (ok) {
       tc_fence_after();
-      __nv_bfloat16* dst = p.dv + ((seq0 + kvc) * p.H + h) * D + qh;
-#pragma unroll 1
-      for (int c = 0; c < 2; c++) {
-        const int nvalid = D - (qh + c * 32);  // columns of this chunk inside d (d = 80: 32, 32, 16, none)
-        if (nvalid <= 0) break;
-        uint32_t v[32];
-        tmem_ld32(tl + C::TM_DV + qh + c * 32, v);
-        tmem_ld_wait(v);
-        if (kv < p.L) {
-          float f[32];
-#pragma unroll
-          for (int e = 0; e < 32; e++) f[e] = __uint_as_float(v[e]);
-          store_row(dst + c * 32, f, nvalid < 32 ? nvalid : 32);
-        }
-      }
-      tc_fence_before();
-      mbar_arrive_warp(&bars->dv_free);  // dV of this item has left TMEM
+      auto release = [&] {
+        tc_fence_before();
+        mbar_arrive_warp(&bars->dv_free);  // dV of this item has left TMEM
+      };
+      if (WALK == kWalkOwned) dv_epilogue<D>(p, tl + C::TM_DV + qh, qh, seq0, h, I.kv0 + 32 * (warp & 3), lane, release);
+      else dv_epilogue_rows<D>(p, tl + C::TM_DV + qh, qh, seq0, h, kv, release);
     }
     g0 += nq;
     }
   } else {
     // ---------------- dQ drain warps 8-11: thread t <-> TMEM lane t <-> column d = t of dQ^T
-    const int t = threadIdx.x - 256;
     const int w = warp & 3;                       // column chunk d = 32 w .. 32 w + 31
     const uint32_t tl = tmem + ((uint32_t)(w * 32) << 16);
     float* stg2 = sSTG + w * (2 * 32 * 32);       // this warp's two [32 q][32] staging slices
@@ -493,20 +481,10 @@ __global__ void __launch_bounds__(512, 1)
     if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&bars->mma_done, ic & 1, wd));
     if (ok) {
       tc_fence_after();
-      const int kv = kv0 + t;
-      const int kvc = kv < p.L ? kv : p.L - 1;
-      __nv_bfloat16* dst = p.dk + ((seq0 + kvc) * p.H + h) * D;
-#pragma unroll 1
-      for (int c = 0; c < C::NCH; c++) {
-        uint32_t v[32];
-        tmem_ld32(tl + C::TM_DK + c * 32, v);
-        tmem_ld_wait(v);
-        // With RoPE, R^T per pair from the warp-coalesced (cos, sin) table.
-        if (kv < p.L)
-          store_dk_row32(dst + c * 32, v, p.scale, p.rope_tab, kv, D, c * 8, D - c * 32 < 32 ? D - c * 32 : 32);
-      }
-      tc_fence_before();
-      mbar_arrive_warp(&bars->dk_free);  // dK of this item has left TMEM
+      dk_epilogue_rows<D, C::NCH>(p, tl + C::TM_DK, seq0, h, kv0 + 32 * w + lane, [&] {
+        tc_fence_before();
+        mbar_arrive_warp(&bars->dk_free);  // dK of this item has left TMEM
+      });
     }
     // dQ owned: the query tiles whose last contributor is this key tile are complete once
     // this warp's copies have landed; convert its chunk of their rows to bf16 dq.
