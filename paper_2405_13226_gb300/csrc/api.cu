@@ -152,9 +152,9 @@ dd_status fwd_common(const dd_attn_desc* desc, const void* q, const void* k, con
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const int nkt = (desc->L + 127) / 128;
   const int rope = !fused_rope ? 0 : (nkt <= kFwdRopeQKMaxTiles ? 2 : 1);  // launch_attn_fwd's RoPE form
-  CUtensorMap tq, tk, tv;
+  CUtensorMap tq, tk, tv, to;
   if (!make_map(&tq, q, desc, 128) || !make_map(&tk, rope == 1 ? k_rot : k, desc, 128) ||
-      !make_map(&tv, v, desc, 128))
+      !make_map(&tv, v, desc, 128) || !make_map(&to, o, desc, 32))  // o: stored in 32-row blocks
     return DD_ERR_CUDA;
   FwdParams p;
   p.B = desc->B;
@@ -192,7 +192,7 @@ dd_status fwd_common(const dd_attn_desc* desc, const void* q, const void* k, con
       if ((e = launch_rope_qk(rp, s)) != cudaSuccess) return DD_ERR_CUDA;
     }
   }
-  e = launch_attn_fwd(desc->d, tq, tk, tv, p, rope, s);
+  e = launch_attn_fwd(desc->d, tq, tk, tv, to, p, rope, s);
   return e == cudaSuccess ? DD_OK : DD_ERR_CUDA;
 }
 

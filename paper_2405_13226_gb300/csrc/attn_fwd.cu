@@ -63,7 +63,9 @@ struct FwdCfg {
   static constexpr int OFF_K = OFF_Q + 2 * Q_BYTES;
   static constexpr int OFF_V = OFF_K + KST * KV_BYTES;
   static constexpr int OFF_BAR = OFF_V + VST * KV_BYTES;
+  static constexpr int OFF_OST = OFF_BAR + 1024;  // RoPE forms: O staging, 4 KB per softmax warp (32 x 64)
   static constexpr int SMEM_BYTES = OFF_BAR + 512 + 1024;
+  static constexpr int SMEM_BYTES_ROPE = OFF_OST + 8 * 4096 + 1024;
   static constexpr int PF = 4;  // K / V tiles prefetched into L2 ahead of the ring
   static constexpr uint32_t TMEM_S = 0, TMEM_O = 256, TMEM_COLS = 512;
   static constexpr int THREADS = 384;  // the RoPE forms add a rotation warpgroup: 512
@@ -229,7 +231,8 @@ __device__ __forceinline__ void rope_rotate_tile(uint8_t* tile, int pos0, int L,
 template <int D, int ROPE>
 __global__ void __launch_bounds__(fwd_threads(ROPE), 1)
     attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
-                       const __grid_constant__ CUtensorMap tmV, const FwdParams p) {
+                    const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmO,
+                    const FwdParams p) {
   using C = FwdCfg<D>;
   constexpr int KST = C::KST, VST = C::VST;
   extern __shared__ uint8_t smem_raw[];
@@ -609,24 +612,66 @@ __global__ void __launch_bounds__(fwd_threads(ROPE), 1)
       mbar_arrive(&bars->v_empty[(jg0 + hi_t - J0) & 1]);
     const float inv_l = l_run > 0.f ? 1.f / l_run : 0.f;
     const float m_use = (m_run == -INFINITY) ? 0.f : m_run;
-    __nv_bfloat16* orow = p.o + (((long long)b * p.L + rowc) * p.H + h) * D;
+    // The RoPE forms: O leaves through shared memory and tensor stores; the plain forward keeps
+    // each thread's own row stores. Measured per forward (H = 16, d = 128, 65536 tokens), tensor
+    // stores made the RoPE forward 12% / 5% faster at L = 256 / 512 (its rotation warpgroup
+    // also stores rows), the plain one 3-4% slower at L = 256 / 512 and 1-2% faster from
+    // L = 4096 and on the concat-and-chunk step; choosing at run time slowed the plain kernel
+    // by 4-6% at L = 512..2048.
+    if constexpr (ROPE != kRopeNone) {
+      // O / l -> bf16 through this warp's 4 KB staging block: its 32 rows x 64 columns in the O
+      // map's 128-byte swizzled layout (16-byte chunk j of row r at r * 128 + ((j ^ (r & 7)) * 16),
+      // conflict-free), then one tensor store per 64 columns, which clips rows past L and
+      // columns past d and writes whole lines (rows are H d elements apart, so each store
+      // instruction of a warp storing its own rows touches 32 lines).
+      const uint32_t ost = smem_u32(smem + C::OFF_OST) + (uint32_t)(t * 4 + (warp & 3)) * 4096u;
+      const int lr = r & 31;  // the thread's row within its warp's 32
 #pragma unroll 1
-    for (int c = 0; c < C::DCH; c++) {
-      uint32_t ov[32];
-      tmem_ld32(obuf + c * 32, ov);
-      tmem_ld_wait(ov);
-      if (row < p.L) {
-        uint4* dst = reinterpret_cast<uint4*>(orow + c * 32);
-        const int nv = (D - c * 32 >= 32) ? 4 : (D - c * 32) / 8;  // 16-byte stores in this chunk
+      for (int hf = 0; hf < C::DB; hf++) {
+        if (lane == 0) bulk_wait_read<0>();  // the previous tensor store has read the block
+        __syncwarp();
+#pragma unroll 1
+        for (int cc = 0; cc < 2 && 2 * hf + cc < C::DCH; cc++) {
+          uint32_t ov[32];
+          tmem_ld32(obuf + (2 * hf + cc) * 32, ov);
+          tmem_ld_wait(ov);
 #pragma unroll
-        for (int q = 0; q < 4; q++) {
-          if (q >= nv) break;
-          uint4 w;
-          w.x = pack_bf16x2(__uint_as_float(ov[8 * q + 0]) * inv_l, __uint_as_float(ov[8 * q + 1]) * inv_l);
-          w.y = pack_bf16x2(__uint_as_float(ov[8 * q + 2]) * inv_l, __uint_as_float(ov[8 * q + 3]) * inv_l);
-          w.z = pack_bf16x2(__uint_as_float(ov[8 * q + 4]) * inv_l, __uint_as_float(ov[8 * q + 5]) * inv_l);
-          w.w = pack_bf16x2(__uint_as_float(ov[8 * q + 6]) * inv_l, __uint_as_float(ov[8 * q + 7]) * inv_l);
-          dst[q] = w;
+          for (int q = 0; q < 4; q++) {
+            const int j = 4 * cc + q;
+            st_shared_v4(ost + lr * 128 + ((j ^ (lr & 7)) << 4),
+                         pack_bf16x2(__uint_as_float(ov[8 * q + 0]) * inv_l, __uint_as_float(ov[8 * q + 1]) * inv_l),
+                         pack_bf16x2(__uint_as_float(ov[8 * q + 2]) * inv_l, __uint_as_float(ov[8 * q + 3]) * inv_l),
+                         pack_bf16x2(__uint_as_float(ov[8 * q + 4]) * inv_l, __uint_as_float(ov[8 * q + 5]) * inv_l),
+                         pack_bf16x2(__uint_as_float(ov[8 * q + 6]) * inv_l, __uint_as_float(ov[8 * q + 7]) * inv_l));
+          }
+        }
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) {
+          tma_store_4d(&tmO, smem + C::OFF_OST + (t * 4 + (warp & 3)) * 4096, 64 * hf, h, row0 + 32 * (warp & 3), b);
+          bulk_commit();
+        }
+      }
+    } else {
+      __nv_bfloat16* orow = p.o + (((long long)b * p.L + rowc) * p.H + h) * D;
+#pragma unroll 1
+      for (int c = 0; c < C::DCH; c++) {
+        uint32_t ov[32];
+        tmem_ld32(obuf + c * 32, ov);
+        tmem_ld_wait(ov);
+        if (row < p.L) {
+          uint4* dst = reinterpret_cast<uint4*>(orow + c * 32);
+          const int nv = (D - c * 32 >= 32) ? 4 : (D - c * 32) / 8;  // 16-byte stores in this chunk
+#pragma unroll
+          for (int q = 0; q < 4; q++) {
+            if (q >= nv) break;
+            uint4 w;
+            w.x = pack_bf16x2(__uint_as_float(ov[8 * q + 0]) * inv_l, __uint_as_float(ov[8 * q + 1]) * inv_l);
+            w.y = pack_bf16x2(__uint_as_float(ov[8 * q + 2]) * inv_l, __uint_as_float(ov[8 * q + 3]) * inv_l);
+            w.z = pack_bf16x2(__uint_as_float(ov[8 * q + 4]) * inv_l, __uint_as_float(ov[8 * q + 5]) * inv_l);
+            w.w = pack_bf16x2(__uint_as_float(ov[8 * q + 6]) * inv_l, __uint_as_float(ov[8 * q + 7]) * inv_l);
+            dst[q] = w;
+          }
         }
       }
     }
@@ -636,6 +681,7 @@ __global__ void __launch_bounds__(fwd_threads(ROPE), 1)
   nit++;
   jg0 += I.NJ;
   }
+  if (ROPE != kRopeNone && lane == 0) bulk_wait<0>();  // this warp's tensor stores of O have landed
   }
 
   tc_fence_before();
@@ -648,11 +694,12 @@ __global__ void __launch_bounds__(fwd_threads(ROPE), 1)
 
 template <int D, int ROPE>
 static cudaError_t launch_fwd_d(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
-                               const FwdParams& p, cudaStream_t stream) {
+                               const CUtensorMap& to, const FwdParams& p, cudaStream_t stream) {
   using C = FwdCfg<D>;
   static DeviceCache nsm_dev;
   int nsm = 0;
-  cudaError_t e = kernel_setup(nsm_dev, attn_fwd_kernel<D, ROPE>, C::SMEM_BYTES, &nsm);
+  constexpr int smem_bytes = ROPE != kRopeNone ? C::SMEM_BYTES_ROPE : C::SMEM_BYTES;
+  cudaError_t e = kernel_setup(nsm_dev, attn_fwd_kernel<D, ROPE>, smem_bytes, &nsm);
   if (e != cudaSuccess) return e;
   // One CTA per SM (shared memory allows no more) walking items: the first G in order, the
   // rest claimed. G is kept coprime with the pairs per (sequence, head), so the first round
@@ -671,23 +718,23 @@ static cudaError_t launch_fwd_d(const CUtensorMap& tq, const CUtensorMap& tk, co
   };
   while (G > 1 && gcd(G, nqp) != 1) G--;
   if ((e = cudaMemsetAsync(p.work_ctr, 0, sizeof(unsigned int), stream)) != cudaSuccess) return e;  // the claim counter
-  attn_fwd_kernel<D, ROPE><<<(unsigned)G, fwd_threads(ROPE), C::SMEM_BYTES, stream>>>(tq, tk, tv, p);
+  attn_fwd_kernel<D, ROPE><<<(unsigned)G, fwd_threads(ROPE), smem_bytes, stream>>>(tq, tk, tv, to, p);
   return cudaGetLastError();
 }
 
 template <int D>
 static cudaError_t launch_fwd_rope(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
-                                   const FwdParams& p, int rope, cudaStream_t stream) {
-  if (rope == kRopeQK) return launch_fwd_d<D, kRopeQK>(tq, tk, tv, p, stream);
-  if (rope == kRopeQ) return launch_fwd_d<D, kRopeQ>(tq, tk, tv, p, stream);
-  return launch_fwd_d<D, kRopeNone>(tq, tk, tv, p, stream);
+                                   const CUtensorMap& to, const FwdParams& p, int rope, cudaStream_t stream) {
+  if (rope == kRopeQK) return launch_fwd_d<D, kRopeQK>(tq, tk, tv, to, p, stream);
+  if (rope == kRopeQ) return launch_fwd_d<D, kRopeQ>(tq, tk, tv, to, p, stream);
+  return launch_fwd_d<D, kRopeNone>(tq, tk, tv, to, p, stream);
 }
 
 cudaError_t launch_attn_fwd(int d, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
-                            const FwdParams& p, int rope, cudaStream_t stream) {
-  if (d == 64) return launch_fwd_rope<64>(tq, tk, tv, p, rope, stream);
-  if (d == 80) return launch_fwd_rope<80>(tq, tk, tv, p, rope, stream);
-  return launch_fwd_rope<128>(tq, tk, tv, p, rope, stream);
+                            const CUtensorMap& to, const FwdParams& p, int rope, cudaStream_t stream) {
+  if (d == 64) return launch_fwd_rope<64>(tq, tk, tv, to, p, rope, stream);
+  if (d == 80) return launch_fwd_rope<80>(tq, tk, tv, to, p, rope, stream);
+  return launch_fwd_rope<128>(tq, tk, tv, to, p, rope, stream);
 }
 
 }  // namespace ddattn

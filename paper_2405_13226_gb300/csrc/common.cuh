@@ -222,7 +222,7 @@ dd_status validate_desc(const dd_attn_desc* desc);
 // Launchers (defined in attn_fwd.cu / attn_bwd.cu / rope.cu); return a cudaError_t.
 // rope: 0 none; 1 the kernel rotates its Q tiles (k given rotated); 2 it rotates Q and K tiles.
 cudaError_t launch_attn_fwd(int d, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
-                            const FwdParams& p, int rope, cudaStream_t stream);
+                            const CUtensorMap& to, const FwdParams& p, int rope, cudaStream_t stream);
 cudaError_t launch_attn_bwd_main_d128(int d, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
                                       const CUtensorMap& tdo, const BwdParams& p, cudaStream_t stream);
 cudaError_t launch_attn_bwd_main_d128_persist(int d, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
