@@ -542,7 +542,8 @@ __global__ void __launch_bounds__(320, 1)
 // slot and write bf16 dq themselves, so the accumulator is neither zeroed (pre) nor converted
 // (post). Measured against the shared accumulator in one process (H = 16, d = 128, 65536
 // tokens): backward 0.742 -> 0.709 ms at L = 256, but 0.912 -> 0.943 at 512, 1.178 -> 1.423
-// at 1024 and 1.642 -> 1.929 at 2048. Per CTA the slot and the re-read window of its pair's
+// at 1024 and 1.642 -> 1.929 at 2048 (at 512 again with the dQ-owned walk's transposed dV
+// epilogue: 0.926 -> 0.950). Per CTA the slot and the re-read window of its pair's
 // Q / dO tiles grow with L (0.5 MB each at L = 1024, times 152 CTAs), so they fall out of L2,
 // while the per-key-tile walk shares each Q / dO tile between the CTAs that work on one pair
 // at the same time; and each pair's conversion holds the drain warps.
